@@ -1,0 +1,322 @@
+"""Pins for the CPU oracle: each check ties the oracle to something other than
+itself -- a library routine, a closed form, an invariant of the method, a
+brute force on tiny inputs or a hand-derived case -- so that a dropped term, a
+wrong sign or index, or a transposed operand in oracle/hill_oracle.c fails at
+least one of them.  CPU only.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2602_18750_gb300 import inputs
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "tiny_cases.json")
+
+
+def _expr(v):
+    return eval(str(v), {"__builtins__": {}}, {"e": math.e, "exp": math.exp})
+
+
+def _exact(oracle_mod, t):
+    return oracle_mod.decode16(t)
+
+
+def _expand_kv(x, H):
+    """[B][Hkv][cap][d] -> [B][H][cap][d] with the contiguous head grouping
+    (query head h reads KV head h // (H/Hkv)), via torch.repeat_interleave."""
+    return torch.repeat_interleave(x, H // x.shape[1], dim=1)
+
+
+# ---------------------------------------------------------------- decoding
+def test_decode_f16_all_bit_patterns(oracle_mod):
+    bits = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    got = oracle_mod.decode16(bits, dtype=oracle_mod.F16)
+    ref = bits.view(np.float16).astype(np.float64)
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(got), nan)
+    assert np.array_equal(got[~nan], ref[~nan])
+
+
+def test_decode_bf16_all_bit_patterns(oracle_mod):
+    bits = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    got = oracle_mod.decode16(bits, dtype=oracle_mod.BF16)
+    ref = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).double().numpy()
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(got), nan)
+    assert np.array_equal(got[~nan], ref[~nan])
+
+
+# ---------------------------------------------------------------- golden
+@pytest.mark.parametrize("case", json.load(open(GOLDEN))["cases"], ids=lambda c: c["name"])
+@pytest.mark.parametrize("dtype", [torch.float16, torch.bfloat16])
+def test_golden_hand_derived(oracle_mod, case, dtype):
+    q = torch.tensor(case["q"], dtype=dtype)
+    K = torch.tensor(case["K"], dtype=dtype)
+    V = torch.tensor(case["V"], dtype=dtype)
+    lens, k, max_k = case["lens"], case["k"], case["max_k"]
+    z = oracle_mod.logits(q, K, lens)
+    for b, n in enumerate(lens):
+        for h in range(case["H"]):
+            want = [_expr(x) for x in case["z"][b][h]]
+            assert np.allclose(z[b, h, :n], want, rtol=0, atol=1e-15)
+            assert np.all(np.isnan(z[b, h, n:]))
+    for mode, key in ((oracle_mod.ATTN, "attn"), (oracle_mod.RAW, "raw")):
+        s = oracle_mod.scores(mode, z, lens)
+        for b, n in enumerate(lens):
+            want = [_expr(x) for x in case[f"s_{key}"][b]]
+            assert np.allclose(s[b, :n], want, rtol=1e-14, atol=1e-15)
+        idx, count, rc = oracle_mod.topk(s, lens, k, max_k)
+        assert rc == 0
+        assert idx.tolist() == case[f"idx_{key}"]
+        assert count.tolist() == case["count"]
+        r = oracle_mod.evict_step(mode, q, K, V, lens, k, max_k)
+        assert r["rc"] == 0 and r["idx"].tolist() == case[f"idx_{key}"]
+        if key == "attn":
+            want = np.array([[[_expr(x) for x in row] for row in hb] for hb in case["out_attn"]])
+            assert np.allclose(r["out"], want, rtol=1e-14, atol=1e-15)
+
+
+# ---------------------------------------------------------------- logits
+@pytest.mark.parametrize("H,Hkv,d", [(8, 8, 128), (8, 2, 64), (4, 1, 128), (6, 3, 32)])
+@pytest.mark.parametrize("dtype", [torch.float16, torch.bfloat16])
+def test_logits_match_torch_fp64_matmul(oracle_mod, H, Hkv, d, dtype):
+    B, cap = 3, 70
+    lens = [70, 33, 0]
+    q, K, V, _ = inputs.random_case(B, H, Hkv, d, cap, lens, dtype=dtype, seed=11)
+    z = oracle_mod.logits(q, K, lens)
+    ref = torch.matmul(_expand_kv(K.double(), H), q.double().unsqueeze(-1)).squeeze(-1) / math.sqrt(d)
+    for b, n in enumerate(lens):
+        assert np.allclose(z[b, :, :n], ref[b, :, :n].numpy(), rtol=1e-12, atol=1e-12)
+        assert np.all(np.isnan(z[b, :, n:]))
+
+
+# ---------------------------------------------------------------- importance
+def test_attn_single_head_is_torch_softmax(oracle_mod):
+    B, H, d, cap = 2, 1, 128, 90
+    lens = [90, 41]
+    q, K, V, _ = inputs.random_case(B, H, H, d, cap, lens, seed=3, kind="zipf")
+    z = oracle_mod.logits(q, K, lens)
+    s = oracle_mod.scores(oracle_mod.ATTN, z, lens)
+    for b, n in enumerate(lens):
+        ref = torch.softmax(torch.from_numpy(z[b, 0, :n]), dim=0).numpy()
+        assert np.allclose(s[b, :n], ref, rtol=1e-12, atol=1e-15)
+
+
+@pytest.mark.parametrize("H,Hkv", [(8, 8), (8, 2), (4, 1)])
+def test_attn_is_sum_of_torch_softmax_rows(oracle_mod, H, Hkv):
+    B, d, cap = 2, 64, 57
+    lens = [57, 19]
+    q, K, V, _ = inputs.random_case(B, H, Hkv, d, cap, lens, seed=5, kind="zipf" if H == Hkv else "normal")
+    z = oracle_mod.logits(q, K, lens)
+    s = oracle_mod.scores(oracle_mod.ATTN, z, lens)
+    for b, n in enumerate(lens):
+        p = torch.softmax(torch.from_numpy(z[b, :, :n]), dim=-1)
+        assert np.allclose(s[b, :n], p.sum(0).numpy(), rtol=1e-12, atol=1e-15)
+        # invariants: every weight is a probability and each head contributes mass 1
+        assert np.isclose(s[b, :n].sum(), H, rtol=1e-12)
+        assert np.all(s[b, :n] >= 0) and np.all(s[b, :n] <= H)
+        assert np.all(np.isnan(s[b, n:]))
+
+
+def test_raw_mqa_closed_form(oracle_mod):
+    """MQA (one KV head): sum_h q_h.K_j/sqrt(d) = (sum_h q_h).K_j/sqrt(d)."""
+    B, H, d, cap = 2, 6, 128, 40
+    lens = [40, 13]
+    q, K, V, _ = inputs.random_case(B, H, 1, d, cap, lens, seed=9)
+    s = oracle_mod.scores(oracle_mod.RAW, oracle_mod.logits(q, K, lens), lens)
+    qx, Kx = _exact(oracle_mod, q), _exact(oracle_mod, K)
+    for b, n in enumerate(lens):
+        ref = Kx[b, 0, :n] @ qx[b].sum(0) / math.sqrt(d)
+        assert np.allclose(s[b, :n], ref, rtol=1e-12, atol=1e-12)
+
+
+def test_raw_gqa_group_sums(oracle_mod):
+    """GQA: RAW importance equals sum over KV heads g of (sum of the G query
+    heads of g) . K_g,j / sqrt(d) -- pins the head -> KV-head map."""
+    B, H, Hkv, d, cap = 1, 8, 2, 32, 25
+    lens = [25]
+    q, K, V, _ = inputs.random_case(B, H, Hkv, d, cap, lens, seed=21)
+    s = oracle_mod.scores(oracle_mod.RAW, oracle_mod.logits(q, K, lens), lens)
+    qx, Kx = _exact(oracle_mod, q), _exact(oracle_mod, K)
+    G = H // Hkv
+    ref = sum(Kx[0, g] @ qx[0, g * G:(g + 1) * G].sum(0) for g in range(Hkv)) / math.sqrt(d)
+    assert np.allclose(s[0], ref, rtol=1e-12, atol=1e-12)
+    # a transposed grouping (h -> h % Hkv) gives a different answer on this input
+    wrong = sum(Kx[0, g] @ qx[0, g::Hkv].sum(0) for g in range(Hkv)) / math.sqrt(d)
+    assert not np.allclose(s[0], wrong, rtol=1e-6)
+
+
+def test_accumulation_mass_over_steps(oracle_mod):
+    """Running importance: after t steps of ATTN, sum_j A[b,j] = H * t."""
+    B, H, d, cap, steps = 2, 4, 64, 30, 5
+    A = np.zeros((B, cap))
+    _, K, V, _ = inputs.random_case(B, H, H, d, cap, [30, 30], seed=2)
+    for t in range(steps):
+        lens = [20 + t, 10 + 2 * t]
+        q = inputs.step_query(inputs.config(2, layers=1, batch=B, heads=H, kv_heads=H, head_dim=d,
+                                            prompt_lens=(20, 10), steps=steps), 0, t)
+        s = oracle_mod.scores(oracle_mod.ATTN, oracle_mod.logits(q, K, lens), lens)
+        A_new = oracle_mod.accumulate(s, A, lens)
+        for b, n in enumerate(lens):
+            assert np.allclose(A_new[b, :n] - A[b, :n], s[b, :n], rtol=0, atol=1e-15)
+            assert np.array_equal(A_new[b, n:], A[b, n:])
+        A = A_new
+    assert np.allclose(A.sum(1), H * steps, rtol=1e-12)
+
+
+# ---------------------------------------------------------------- top-k
+def _brute_topk(key, n, k):
+    order = sorted(range(n), key=lambda j: (-key[j], j))
+    return sorted(order[: max(0, min(k, n))])
+
+
+def test_topk_brute_force_and_torch_values(oracle_mod):
+    rng = np.random.default_rng(0)
+    B, cap = 6, 64
+    key = rng.standard_normal((B, cap))
+    key[1, 10:20] = 0.5                      # a block of exact ties
+    key[2] = np.round(key[2])                # heavy ties
+    lens = [64, 40, 64, 1, 0, 17]
+    k = [13, 15, 30, 5, 3, 17]
+    max_k = 32
+    idx, count, rc = oracle_mod.topk(key, lens, k, max_k)
+    assert rc == 0
+    for b in range(B):
+        want = _brute_topk(key[b], lens[b], k[b])
+        assert count[b] == len(want) == min(k[b], lens[b])
+        assert idx[b, : count[b]].tolist() == want
+        assert np.all(idx[b, count[b]:] == -1)
+        if lens[b] and k[b]:
+            tv = torch.topk(torch.from_numpy(key[b, : lens[b]]), min(k[b], lens[b])).values
+            assert sorted(key[b, want].tolist()) == sorted(tv.tolist())
+
+
+def test_topk_special_budgets(oracle_mod):
+    rng = np.random.default_rng(1)
+    key = rng.standard_normal((3, 50))
+    lens = [50, 50, 30]
+    idx, count, rc = oracle_mod.topk(key, lens, [50, 0, 99], 50)
+    assert rc == 0
+    assert idx[0].tolist() == list(range(50))           # k = len: everything
+    assert count[1] == 0 and np.all(idx[1] == -1)       # k = 0: nothing
+    assert idx[2, :30].tolist() == list(range(30))      # k > len clamps to len
+    idx, count, rc = oracle_mod.topk(key, lens, [40, 40, 40], 8)
+    assert rc == 2 and count.tolist() == [8, 8, 8]      # capped by max_k, reported
+
+
+def test_topk_ties_go_to_lower_index(oracle_mod):
+    key = np.zeros((1, 12))
+    key[0, [3, 7, 9]] = 2.0
+    idx, count, _ = oracle_mod.topk(key, [12], [5], 5)
+    assert idx[0].tolist() == [0, 1, 3, 7, 9]
+    key[0, 5] = -0.0                         # signed zero ties with +0
+    idx, count, _ = oracle_mod.topk(key, [12], [5], 5)
+    assert idx[0].tolist() == [0, 1, 3, 7, 9]
+
+
+def test_topk_nan_ranks_last(oracle_mod):
+    key = np.array([[np.nan, 1.0, -5.0, np.nan, 0.0]])
+    idx, count, _ = oracle_mod.topk(key, [5], [3], 5)
+    assert idx[0, :3].tolist() == [1, 2, 4]
+
+
+def test_cec_single_head_raw_equals_attn_selection(oracle_mod):
+    """Sec. 4.4: for one head and one step, ranking by raw q.K equals ranking by
+    softmax weight (softmax is monotonic), so both modes select the same set."""
+    for seed in range(4):
+        q, K, V, _ = inputs.random_case(2, 1, 1, 128, 300, [300, 257], seed=seed, kind="zipf")
+        lens, k = [300, 257], [60, 25]
+        ra = oracle_mod.evict_step(oracle_mod.ATTN, q, K, V, lens, k, 64, with_attn=False)
+        rr = oracle_mod.evict_step(oracle_mod.RAW, q, K, V, lens, k, 64, with_attn=False)
+        assert np.array_equal(ra["idx"], rr["idx"])
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_planted_heavy_hitters_always_selected(oracle_mod, mode):
+    """The heavy-hitter workload (64 planted keys, 4x along q) at reduced size:
+    every planted token is in the selected set in both modes."""
+    w = inputs.config(1, heads=4, kv_heads=4, prompt_lens=(512,), planted=16, budget_tokens=64)
+    K, V = inputs.layer_cache(w, 0)
+    q = inputs.step_query(w, 0, 0)
+    # recover the planted positions from the generator's construction: their
+    # projection on the query direction is 4*sqrt(d) for every head
+    qx = oracle_mod.decode16(q)[0]
+    Kx = oracle_mod.decode16(K)[0]
+    proj = np.stack([Kx[h] @ (qx[h] / np.linalg.norm(qx[h])) for h in range(4)])
+    planted = np.where((proj > 2.0 * math.sqrt(128)).all(0))[0]
+    assert len(planted) == 16
+    r = oracle_mod.evict_step(mode, q, K, V, [512], [64], 64, with_attn=False)
+    assert set(planted.tolist()) <= set(r["idx"][0, : r["count"][0]].tolist())
+
+
+# ---------------------------------------------------------------- attention
+@pytest.mark.parametrize("H,Hkv", [(8, 8), (8, 2), (4, 1)])
+@pytest.mark.parametrize("dtype", [torch.float16, torch.bfloat16])
+def test_full_budget_equals_dense_sdpa(oracle_mod, H, Hkv, dtype):
+    """k = len selects every token, so the sparse attention is the dense decode
+    attention: torch scaled_dot_product_attention in float64."""
+    B, d, cap = 2, 64, 45
+    lens = [45, 22]
+    q, K, V, _ = inputs.random_case(B, H, Hkv, d, cap, lens, dtype=dtype, seed=4)
+    r = oracle_mod.evict_step(oracle_mod.ATTN, q, K, V, lens, lens, cap)
+    Ke, Ve = _expand_kv(K.double(), H), _expand_kv(V.double(), H)
+    for b, n in enumerate(lens):
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            q[b].double().unsqueeze(1), Ke[b, :, :n], Ve[b, :, :n]).squeeze(1)
+        assert np.allclose(r["out"][b], ref.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_attention_special_cases(oracle_mod):
+    B, H, Hkv, d, cap = 2, 4, 2, 32, 20
+    q, K, V, _ = inputs.random_case(B, H, Hkv, d, cap, [20, 20], seed=8)
+    Vx = oracle_mod.decode16(V)
+    # one selected token: the output is exactly that token's value row
+    idx = np.array([[7], [13]], dtype=np.int32)
+    out = oracle_mod.sparse_attn(q, K, V, idx, [1, 1])
+    for b in range(B):
+        for h in range(H):
+            assert np.array_equal(out[b, h], Vx[b, h // 2, idx[b, 0]])
+    # a constant value cache gives that constant whatever the weights
+    Vc = torch.full_like(V, 1.5)
+    idx = np.array([[0, 3, 9, 19], [2, 4, 6, 8]], dtype=np.int32)
+    out = oracle_mod.sparse_attn(q, K, Vc, idx, [4, 3])
+    assert np.allclose(out, 1.5, rtol=0, atol=1e-15)
+    # empty selection gives zero
+    out = oracle_mod.sparse_attn(q, K, V, idx, [0, 0])
+    assert np.all(out == 0)
+    # the order of the index list does not matter
+    a = oracle_mod.sparse_attn(q, K, V, idx, [4, 4])
+    b = oracle_mod.sparse_attn(q, K, V, idx[:, ::-1].copy(), [4, 4])
+    assert np.allclose(a, b, rtol=1e-14, atol=1e-15)
+
+
+def test_attention_rejects_out_of_range_index(oracle_mod):
+    q, K, V, _ = inputs.random_case(1, 2, 2, 16, 10, [10], seed=1)
+    with pytest.raises(ValueError):
+        oracle_mod.sparse_attn(q, K, V, np.array([[3, 10]], dtype=np.int32), [2])
+
+
+# ---------------------------------------------------------------- planted mistakes
+def test_pins_catch_planted_mistakes(oracle_mod):
+    """Plant plausible mistakes on the CPU side (wrong scale, transposed
+    operand, softmax over the wrong range) and check that the same pins used
+    above reject them."""
+    B, H, d, cap = 1, 4, 64, 30
+    lens = [21]
+    q, K, V, _ = inputs.random_case(B, H, H, d, cap, lens, seed=6)
+    z = oracle_mod.logits(q, K, lens)
+    ref = torch.matmul(K.double(), q.double().unsqueeze(-1)).squeeze(-1) / math.sqrt(d)
+    assert np.allclose(z[0, :, :21], ref[0, :, :21].numpy())
+    # missing 1/sqrt(d)
+    assert not np.allclose(z[0, :, :21] * math.sqrt(d), ref[0, :, :21].numpy())
+    # K read with query and key roles swapped across heads
+    zt = oracle_mod.logits(q.flip(1), K, lens)
+    assert not np.allclose(zt[0, :, :21], ref[0, :, :21].numpy())
+    # softmax over the full capacity instead of the causal row breaks the mass invariant
+    zc = np.where(np.isnan(z), 0.0, z)
+    s_bad = oracle_mod.scores(oracle_mod.ATTN, zc, [cap])
+    assert not np.isclose(s_bad[0, :21].sum(), H)
