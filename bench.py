@@ -1,0 +1,548 @@
+#!/usr/bin/env python
+"""Benchmark of the per-decode-step token-importance evaluation (HillInfer,
+arxiv 2602.18750) on GB300.
+
+One benchmark step is one decode step of the whole stack: for each of the 32
+layers, one hill_evict_step call (score every cached key, aggregate per token
+over heads, select the top-k per sequence, sparse decode attention over the
+selection).  The default workload is the Qwen-7B-shaped stack: 32 layers,
+batch 8, 32 heads MHA, head_dim 128, 4096 -> 4159 cached tokens over 64
+decode steps, budget k = floor(0.2 * len), fp16, ATTN importance.  Inputs are
+synthetic (seeded Zipf(1.1) attention skew) and resident in HBM; every
+layer's K cache (272 MB) is larger than L2 and the 32 layers are distinct, so
+no L2 flush is needed between steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  With N > 1 (torchrun, one rank per GPU) every
+rank runs its own replica of the workload on its own sequences (weak
+scaling); the only collectives are the timing barrier and the max-reduction
+of the elapsed time.  ``--impl reference`` times the CPU oracle on the host
+cores on the same workload and metric.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+from paper_2602_18750_gb300 import inputs  # noqa: E402
+
+METRIC = "cached tokens scored+selected/sec"
+UNIT = "tokens/s"
+L2_BYTES = 129 * 1024 * 1024
+
+
+# ---------------------------------------------------------------- distributed helpers
+def dist_env():
+    """(rank, world, local_rank) from the torchrun environment (1 process if unset)."""
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", str(rank)))
+    return rank, world, local
+
+
+def replica_seed(base_seed: int, rank: int) -> int:
+    """Each rank evaluates its own sequences: a distinct seed per replica."""
+    return base_seed + 1000003 * rank
+
+
+def max_over_ranks(value: float, device=None) -> float:
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(device=None):
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        if device is not None and device.type == "cuda":
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+# ---------------------------------------------------------------- clocks
+def smi_device_id(local: int) -> str:
+    """The nvidia-smi identifier of CUDA device `local` (its UUID when torch
+    exposes it, so that CUDA_VISIBLE_DEVICES remapping cannot point elsewhere)."""
+    try:
+        u = str(torch.cuda.get_device_properties(local).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        if vis:
+            return vis.split(",")[local].strip()
+        return str(local)
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons, each stamped on arrival."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str, period_ms: int = 50):
+        self.samples = []
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-i", gpu_id, "-lms", str(period_ms)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), [x.strip() for x in line.split(",")]))
+
+    def wait_first(self, timeout=3.0):
+        t0 = time.time()
+        while self.proc is not None and not self.samples and time.time() - t0 < timeout:
+            time.sleep(0.02)
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=2)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        inside = [s for t, s in self.samples if t0 <= t <= t1 + 0.05]
+        note = None
+        if not inside:   # a very short timed region: take the samples nearest to it
+            near = sorted(self.samples, key=lambda ts: abs(ts[0] - (t0 + t1) / 2))[:3]
+            inside = [s for _, s in near]
+            note = "no sample inside the timed window; nearest samples used"
+        names = ["active", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(s[0]) for s in inside if num(s[0]) is not None]
+        mx = [num(s[1]) for s in inside if num(s[1]) is not None]
+        pw = [num(s[2]) for s in inside if num(s[2]) is not None]
+        reasons = set()
+        for s in inside:
+            for name, v in zip(names[1:], s[4:8]):
+                if v.strip().lower() == "active":
+                    reasons.add(name)
+        out = {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+               "power_w_max": max(pw) if pw else None, "reasons": sorted(reasons), "samples": len(inside)}
+        if note:
+            out["note"] = note
+        return out
+
+
+# ---------------------------------------------------------------- helpers
+def source_digest(path: str) -> str:
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def profile_traffic(kernel_key: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    the current source of the kernel (else None)."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    digest = source_digest(os.path.join(ROOT, "paper_2602_18750_gb300", "csrc", "score.cu"))
+    for line in open(path):
+        m = re.match(r"\s*(\S+)\s+(\S+)\s+src=(\w+)\s+dram_bytes_per_launch=(\d+)", line)
+        if m and m.group(1) == kernel_key and m.group(2) == workload and m.group(3) == digest:
+            return int(m.group(4))
+    return None
+
+
+def workload_for(n: int, seed: int, layers_resident: int | None):
+    w = inputs.config(n, seed=seed)
+    lres = w.layers
+    if layers_resident:
+        lres = min(lres, layers_resident)
+    return w, lres
+
+
+def describe(w, lres, mode_name):
+    lens0, lens1 = w.lens_at(0), w.lens_at(w.steps - 1)
+    return {
+        "workload": w.name,
+        "layers": w.layers, "layers_resident": lres, "batch": w.batch, "heads": w.heads,
+        "kv_heads": w.kv_heads, "head_dim": w.head_dim,
+        "tokens_first_step": lens0, "tokens_last_step": lens1, "decode_steps": w.steps,
+        "budget": (f"floor({w.budget_frac}*len)" if w.budget_tokens is None else w.budget_tokens),
+        "kv_dtype": str(w.dtype).replace("torch.", ""), "skew": w.kind, "importance": mode_name,
+        "accumulate": w.accumulate,
+        "l2": "inputs larger than L2 (each layer's K > 129 MB; layers distinct), no flush",
+    }
+
+
+# ---------------------------------------------------------------- our implementation
+def run_ours(args):
+    import torch.distributed as dist
+
+    from paper_2602_18750_gb300 import build as hbuild
+    from paper_2602_18750_gb300 import hill
+
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    hbuild.build()
+    hill.load()
+
+    mode = hill.HILL_SCORE_ATTN if args.mode == "attn" else hill.HILL_SCORE_RAW
+    w, lres = workload_for(args.workload, replica_seed(args.seed, rank), args.layers_resident)
+    L, S, B, Hq, Hkv, d = w.layers, w.steps, w.batch, w.heads, w.kv_heads, w.head_dim
+    cap, max_k = w.capacity, w.max_k
+
+    # ---------------- resident inputs: caches, queries, lengths, budgets
+    t_gen = time.time()
+    Kall = torch.empty(lres, B, Hkv, cap, d, dtype=w.dtype, device=dev)
+    Vall = torch.empty_like(Kall)
+    for l in range(lres):
+        K, V = inputs.layer_cache(w, l, device=dev)
+        Kall[l].copy_(K)
+        Vall[l].copy_(V)
+        del K, V
+    q_all = torch.empty(S, L, B, Hq, d, dtype=w.dtype, device=dev)
+    for t in range(S):
+        for l in range(L):
+            q_all[t, l].copy_(inputs.step_query(w, l, t, device=dev))
+    lens_all = torch.tensor([w.lens_at(t) for t in range(S)], dtype=torch.int32, device=dev)
+    k_all = torch.tensor([w.budget_at(t) for t in range(S)], dtype=torch.int32, device=dev)
+    accum = torch.zeros(lres, B, cap, dtype=torch.float32, device=dev) if w.accumulate else None
+    torch.cuda.synchronize()
+    t_gen = time.time() - t_gen
+
+    scores = torch.empty(L, B, cap, dtype=torch.float32, device=dev)
+    idx = torch.empty(L, B, max_k, dtype=torch.int32, device=dev)
+    count = torch.empty(L, B, dtype=torch.int32, device=dev)
+    out = torch.empty(L, B, Hq, d, dtype=torch.float32, device=dev)
+    desc = hill.make_desc(q_all[0, 0], Kall[0], Vall[0])
+    ws = hill.alloc_workspace(desc, mode, max_k, dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def issue_step(t, st):
+        for l in range(L):
+            r = l % lres
+            hill.hill_evict_step(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], max_k, mode,
+                                 accum[r] if accum is not None else None, scores[l], idx[l], count[l],
+                                 out[l], ws, st)
+
+    # eager warm-up of every kernel shape, then one CUDA graph per decode step
+    with torch.cuda.stream(stream):
+        issue_step(0, stream)
+    hill.hill_sync_status(stream)
+    graphs, launches = [], []
+    for t in range(S):
+        g = torch.cuda.CUDAGraph()
+        n0 = hill.hill_kernel_launches()
+        with torch.cuda.graph(g, stream=stream):
+            issue_step(t, stream)
+        launches.append(hill.hill_kernel_launches() - n0)
+        graphs.append(g)
+    if accum is not None:
+        accum.zero_()
+
+    tokens_of = [L * sum(w.lens_at(t)) for t in range(S)]
+    order = [(args.warmup + i) % S for i in range(args.steps)]
+
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            graphs[i % S].replay()
+    stream.synchronize()
+    hill.hill_sync_status(stream)
+
+    # ---------------- timed region (device-resident inputs)
+    clocks = ClockSampler(smi_device_id(local))
+    clocks.wait_first()
+    barrier(dev)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    w0 = time.time()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for t in order:
+            graphs[t].replay()
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    w1 = time.time()
+    barrier(dev)
+    ms_local = e0.elapsed_time(e1)
+    clock_info = clocks.summary(w0, w1)
+    clocks.stop()
+    hill.hill_sync_status(stream)
+    ms = max_over_ranks(ms_local, dev)
+    tokens = sum(tokens_of[t] for t in order)
+    value = world * tokens / (ms / 1e3)
+    k_bytes_per_token = Hkv * d * 2
+    k_gbs = world * tokens * k_bytes_per_token / (ms / 1e3) / 1e9
+    gpu_launches = sum(launches[t] for t in order)
+
+    # ---------------- scoring stage alone, per launch (roofline of the dominant kernels)
+    t_s = S - 1
+    lens_s = w.lens_at(t_s)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(L)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(L)]
+    with torch.cuda.stream(stream):
+        for rep in range(2):
+            for l in range(L):
+                r = l % lres
+                if rep == 1:
+                    starts[l].record(stream)
+                hill.hill_score(desc, q_all[t_s, l], Kall[r], lens_all[t_s], mode, scores[l], None, ws, stream)
+                if rep == 1:
+                    ends[l].record(stream)
+    stream.synchronize()
+    score_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / L
+    # also the whole fused step of one layer (eval-step time per layer)
+    step_us_per_layer = ms_local * 1e3 / (len(order) * L)
+    score_tokens = sum(lens_s)
+    alg_bytes = score_tokens * (k_bytes_per_token + 4) + B * Hq * d * 2
+    peak, peak_kind = measured_peaks()
+    achieved = alg_bytes / (score_ms / 1e3) / 1e9
+    roofline = {
+        "kernel": "hill_score: hill_score_kernel + hill_attn_finalize_kernel" if mode == 0
+        else "hill_score: hill_score_kernel",
+        "bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+        "frac": round(achieved / peak, 4), "peak_source": peak_kind,
+        "traffic": profile_traffic("hill_score_" + args.mode, w.name),
+        "algorithmic_bytes_per_launch": alg_bytes,
+        "bytes_per_token": f"Hkv*d*2 + 4 = {k_bytes_per_token + 4}",
+        "launch_us": round(score_ms * 1e3, 2),
+    }
+
+    # ---------------- end to end through the C ABI with host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all, accum, scores,
+                      idx, count, out, ws, stream, dev, world)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, lres, Kall, Vall, q_all, mode, seconds=args.cpu_seconds)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(ms / len(order), 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f16" if w.dtype == torch.float16 else "bf16",
+            "data": "synthetic", "config": describe(w, lres, args.mode),
+            "k_stream_gbs": round(k_gbs, 1),
+            "k_stream_frac_of_measured_hbm": round(k_gbs / world / peak, 4),
+            "k_stream_frac_of_8tbs": round(k_gbs / world / 8000.0, 4),
+            "eval_step_us_per_layer": round(step_us_per_layer, 2),
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": gpu_launches,
+            "clocks": clock_info, "generate_s": round(t_gen, 1),
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all, accum, scores, idx, count,
+            out, ws, stream, dev, world):
+    """Same steps through hill_evict_step (eager calls), with each step's inputs
+    copied from pinned host memory (query of every layer, the new token's K/V
+    row of every layer, lengths, budgets) and its results (selection and
+    attention output of every layer) copied back, all inside the timed region."""
+    L, S, B = w.layers, w.steps, w.batch
+    order = [(args.warmup + i) % S for i in range(args.steps)]
+    # host copies of what a caller would hold at each step
+    q_h = torch.empty_like(q_all, device="cpu").pin_memory()
+    q_h.copy_(q_all)
+    pos = [[n - 1 for n in w.lens_at(t)] for t in range(S)]
+    newk_h = torch.empty(S, lres, B, w.kv_heads, w.head_dim, dtype=w.dtype).pin_memory()
+    newv_h = torch.empty_like(newk_h).pin_memory()
+    for t in range(S):
+        for b in range(B):
+            newk_h[t, :, b].copy_(Kall[:, b, :, pos[t][b]])
+            newv_h[t, :, b].copy_(Vall[:, b, :, pos[t][b]])
+    lk_h = torch.stack([lens_all.cpu(), k_all.cpu()], 1).pin_memory()        # [S][2][B]
+    lk_d = torch.empty(2, B, dtype=torch.int32, device=dev)
+    stage_k = torch.empty(lres, B, w.kv_heads, w.head_dim, dtype=w.dtype, device=dev)
+    stage_v = torch.empty_like(stage_k)
+    idx_h = torch.empty_like(idx, device="cpu").pin_memory()
+    cnt_h = torch.empty_like(count, device="cpu").pin_memory()
+    out_h = torch.empty_like(out, device="cpu").pin_memory()
+    uniform = [len(set(p)) == 1 for p in pos]
+
+    def one(t):
+        q_all[t].copy_(q_h[t], non_blocking=True)
+        stage_k.copy_(newk_h[t], non_blocking=True)
+        stage_v.copy_(newv_h[t], non_blocking=True)
+        lk_d.copy_(lk_h[t], non_blocking=True)
+        if uniform[t]:
+            Kall[:, :, :, pos[t][0]].copy_(stage_k)
+            Vall[:, :, :, pos[t][0]].copy_(stage_v)
+        else:
+            for b in range(B):
+                Kall[:, b, :, pos[t][b]].copy_(stage_k[:, b])
+                Vall[:, b, :, pos[t][b]].copy_(stage_v[:, b])
+        for l in range(L):
+            r = l % lres
+            hill.hill_evict_step(desc, q_all[t, l], Kall[r], Vall[r], lk_d[0], lk_d[1], w.max_k, mode,
+                                 accum[r] if accum is not None else None, scores[l], idx[l], count[l], out[l],
+                                 ws, stream)
+        idx_h.copy_(idx, non_blocking=True)
+        cnt_h.copy_(count, non_blocking=True)
+        out_h.copy_(out, non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            one(i % S)
+    stream.synchronize()
+    barrier(dev)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for t in order:
+            one(t)
+        e1.record(stream)
+    stream.synchronize()
+    barrier(dev)
+    hill.hill_sync_status(stream)
+    ms = max_over_ranks(e0.elapsed_time(e1), dev)
+    tokens = sum(L * sum(w.lens_at(t)) for t in order)
+    h2d = (q_h[0].numel() * q_h.element_size() + 2 * newk_h[0].numel() * newk_h.element_size()
+           + lk_h[0].numel() * 4)
+    d2h = idx_h.numel() * 4 + cnt_h.numel() * 4 + out_h.numel() * 4
+    return {"value": round(world * tokens / (ms / 1e3), 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": round(ms / len(order), 4),
+            "api": "hill_evict_step per layer, eager (no graph)"}
+
+
+def cpu_baseline(w, lres, Kall, Vall, q_all, mode, seconds=10.0):
+    """The oracle as it stands on the host cores, on (layer, step) samples of
+    the same workload until about `seconds` of CPU time have run."""
+    import oracle
+    oracle.build()
+    done_tokens, spent, samples = 0, 0.0, []
+    for i in range(w.layers * w.steps):
+        l, t = i % w.layers, (i * 7) % w.steps
+        r = l % lres
+        lens, k = w.lens_at(t), w.budget_at(t)
+        q = q_all[t, l].cpu()
+        K, V = Kall[r].cpu(), Vall[r].cpu()
+        t0 = time.perf_counter()
+        oracle.evict_step(mode, q, K, V, lens, k, w.max_k, with_attn=True)
+        spent += time.perf_counter() - t0
+        done_tokens += sum(lens)
+        samples.append(f"L{l}/t{t}")
+        if spent >= seconds:
+            break
+    return {"value": round(done_tokens / spent, 1), "unit": UNIT, "cores": oracle.num_threads(),
+            "kind": "oracle",
+            "sample": f"{len(samples)} (layer, decode step) evaluations of the same workload "
+                      f"({', '.join(samples[:4])}{', ...' if len(samples) > 4 else ''}), all {w.batch} "
+                      f"sequences, score + top-k + sparse attention in float64, {spent:.1f} s"}
+
+
+# ---------------------------------------------------------------- reference arm (the oracle)
+def run_reference(args):
+    """The oracle on the host cores, as it stands: each step is one (layer,
+    decode step) evaluation of the workload (all sequences)."""
+    import oracle
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    oracle.build()
+    w, lres = workload_for(args.workload, args.seed, args.layers_resident)
+    lres = min(lres, 2)   # a couple of distinct layers, generated on the host
+    caches = [inputs.layer_cache(w, l, device="cpu") for l in range(lres)]
+    mode = oracle.ATTN if args.mode == "attn" else oracle.RAW
+
+    def step(i):
+        l, t = i % w.layers, i % w.steps
+        K, V = caches[l % lres]
+        q = inputs.step_query(w, l, t, device="cpu")
+        lens, k = w.lens_at(t), w.budget_at(t)
+        oracle.evict_step(mode, q, K, V, lens, k, w.max_k, with_attn=True)
+        return sum(lens)
+
+    for i in range(args.warmup):
+        step(i)
+    t0 = time.perf_counter()
+    tokens = 0
+    for i in range(args.steps):
+        tokens += step(args.warmup + i)
+    sec = time.perf_counter() - t0
+    value = tokens / sec
+    cores = oracle.num_threads()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(sec * 1e3 / args.steps, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": describe(w, lres, args.mode),
+        "cpu_baseline": {"value": round(value, 1), "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": "each step: one (layer, decode step) of the workload, all "
+                                   f"{w.batch} sequences, score + top-k + sparse attention"},
+        "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=64)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", type=int, default=2, help="1..5 (default 2, the Qwen-7B stack)")
+    ap.add_argument("--mode", choices=["attn", "raw"], default="attn")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--layers-resident", type=int, default=None,
+                    help="allocate this many layers and cycle them (workloads larger than HBM)")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3 and args.impl == "ours":
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

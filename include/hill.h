@@ -1,0 +1,149 @@
+/*
+ * hill.h -- C ABI of libhill.so: GB300 (sm_103a) kernels for the per-decode-
+ * step token-importance evaluation of HillInfer (arxiv 2602.18750).
+ *
+ * One decode step of one layer: score the current query against every cached
+ * key (Eq. 1, Sec. 2.1), aggregate the scores per token over all query heads
+ * (Sec. 4.1 column-sum of attention weights, or the raw inner product of
+ * Sec. 4.4), optionally add them to a running per-token importance, select
+ * the top-k tokens per sequence (Sec. 3.1, Sec. 4.2), and run the decode
+ * attention over the selected tokens only (Sec. 3.1, step 6).
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - All tensor pointers are DEVICE pointers owned by the caller; the library
+ *   never allocates, frees or retains them.  Scratch space comes from the
+ *   caller's workspace `ws` (size from hill_workspace_bytes; 16-byte aligned;
+ *   its contents need no initialisation and are not preserved between calls).
+ * - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
+ *   stream).  A returned HILL_OK means the work was enqueued.  Two calls that
+ *   share a workspace must be ordered on the GPU (same stream).
+ * - Host-side validation failures return immediately and launch nothing.
+ *   Launch failures return HILL_ERR_CUDA.  Conditions only visible on the
+ *   device (a budget larger than max_k, a selected index outside the cache, a
+ *   copy that never completed) set a device error word; hill_sync_status()
+ *   reports and clears it.  No kernel traps or spins without a bound.
+ * - Layouts (element strides, the head dimension contiguous):
+ *     q        [B][H][d]          strides q_sb, q_sh
+ *     k_cache  [B][Hkv][cap][d]   strides k_sb, k_sh, k_sn
+ *     v_cache  [B][Hkv][cap][d]   strides v_sb, v_sh, v_sn
+ *     lens, k, count  [B] int32;  scores, accum  [B][cap] float32 (row = cap);
+ *     idx      [B][max_k] int32;  out  [B][H][d] float32, contiguous.
+ *   Every stride must be a multiple of 8 elements and q/k/v 16-byte aligned.
+ *   Query head h reads KV head h / (H / Hkv) (contiguous grouping).
+ * - lens[b] counts the cached tokens of sequence b including the token
+ *   generated this step (the caller appends its K/V first); it is clamped to
+ *   [0, cap] on the device.  Entries of scores/accum at j >= lens[b] are not
+ *   touched.  k[b] is clamped to [0, lens[b]].
+ * - Supported: head_dim 128; H / Hkv in {1, 2, 4, 8}; fp16 or bf16 q/K/V.
+ */
+#ifndef HILL_H_
+#define HILL_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  HILL_OK = 0,
+  HILL_ERR_INVALID_ARG = 1,  /* bad pointer, size, stride or alignment       */
+  HILL_ERR_UNSUPPORTED = 2,  /* valid but not built (head_dim, group size)    */
+  HILL_ERR_WORKSPACE = 3,    /* ws NULL or smaller than hill_workspace_bytes */
+  HILL_ERR_CUDA = 4,         /* a CUDA runtime call or launch failed          */
+  HILL_ERR_TIMEOUT = 5,      /* a bounded device wait expired (device word)   */
+  HILL_ERR_DEVICE = 6        /* a device-side argument check fired (device word) */
+} hill_status;
+
+typedef enum { HILL_F16 = 0, HILL_BF16 = 1 } hill_dtype;
+
+/* Importance rule.  ATTN (the paper's definition, Sec. 4.1): per (b, h) the
+ * softmax of z = q.K/sqrt(d) over j < lens[b], summed over all H query heads.
+ * RAW (Sec. 4.4 "Algorithmic Simplification"): the sum over heads of z itself
+ * (no softmax); the 1/sqrt(d) scale is kept. */
+typedef enum { HILL_SCORE_ATTN = 0, HILL_SCORE_RAW = 1 } hill_score_mode;
+
+typedef struct {
+  int32_t batch;         /* B  >= 0                                   */
+  int32_t num_q_heads;   /* H  >= 1                                   */
+  int32_t num_kv_heads;  /* Hkv >= 1, H % Hkv == 0                    */
+  int32_t head_dim;      /* d (128)                                   */
+  int32_t capacity;      /* cap: allocated tokens per (b, kv head)    */
+  int32_t dtype;         /* hill_dtype of q, K and V                  */
+  int64_t q_sb, q_sh;             /* element strides of q             */
+  int64_t k_sb, k_sh, k_sn;       /* element strides of k_cache       */
+  int64_t v_sb, v_sh, v_sn;       /* element strides of v_cache       */
+} hill_desc;
+
+/* Bytes of workspace that any call below needs for this descriptor, mode and
+ * index width (the maximum over the four calls).  Returns 0 for an invalid
+ * descriptor.  Queries the current device's SM count. */
+size_t hill_workspace_bytes(const hill_desc* desc, hill_score_mode mode, int32_t max_k);
+
+/* Per-token importance (Eq. 1 with Sec. 4.1 or Sec. 4.4):
+ *   ATTN: scores[b][j] = sum_h softmax_{j'<lens[b]}(q_h . K_{g(h),j'} / sqrt(d))[j]
+ *   RAW : scores[b][j] = sum_h q_h . K_{g(h),j} / sqrt(d)
+ * for j < lens[b].  If accum != NULL it is also updated: accum[b][j] +=
+ * scores[b][j] (running importance across decode steps; a newly appended
+ * token must hold 0 in accum before its first step).  scores is required. */
+hill_status hill_score(const hill_desc* desc, const void* q, const void* k_cache,
+                       const int32_t* lens, hill_score_mode mode, float* scores,
+                       float* accum, void* ws, size_t ws_bytes, void* stream);
+
+/* Top-k selection (Sec. 3.1 top-alpha retention, Sec. 4.2 global top-alpha):
+ * for each b, the first n_b = min(k[b], lens[b]) tokens j < lens[b] in the
+ * order (scores[b][j] descending, j ascending) -- a lower index wins a tie --
+ * written to idx[b][0..n_b) in ascending index order, idx[b][n_b..max_k) =
+ * -1, count[b] = n_b.  If n_b > max_k, count[b] = max_k and the device error
+ * word records HILL_ERR_DEVICE.  -0.0 ranks equal to +0.0; keys must be
+ * finite. */
+hill_status hill_topk_select(const hill_desc* desc, const float* scores, const int32_t* lens,
+                             const int32_t* k, int32_t max_k, int32_t* idx, int32_t* count,
+                             void* ws, size_t ws_bytes, void* stream);
+
+/* Decode attention over the selected tokens only (Sec. 3.1 step 6; Eq. 1
+ * restricted to the selected set, softmax renormalised over it):
+ *   out[b][h][:] = sum_{t<count[b]} p_t V[b][g(h)][idx[b][t]][:],
+ *   p = softmax_t(q_h . K[b][g(h)][idx[b][t]] / sqrt(d)).
+ * count[b] == 0 gives zeros.  count[b] is clamped to [0, max_k]; an index
+ * outside [0, cap) is skipped and recorded as HILL_ERR_DEVICE. */
+hill_status hill_gather_sparse_attn(const hill_desc* desc, const void* q, const void* k_cache,
+                                    const void* v_cache, const int32_t* idx, const int32_t* count,
+                                    int32_t max_k, float* out, void* ws, size_t ws_bytes,
+                                    void* stream);
+
+/* The whole step for one layer: hill_score, then hill_topk_select on accum
+ * (if given) else on this step's scores, then (if out != NULL)
+ * hill_gather_sparse_attn over the selection.  scores may be NULL (then the
+ * step's scores live in the workspace).  Results equal those of the three
+ * separate calls. */
+hill_status hill_evict_step(const hill_desc* desc, const void* q, const void* k_cache,
+                            const void* v_cache, const int32_t* lens, const int32_t* k,
+                            int32_t max_k, hill_score_mode mode, float* accum, float* scores,
+                            int32_t* idx, int32_t* count, float* out, void* ws,
+                            size_t ws_bytes, void* stream);
+
+/* Synchronises `stream`, then returns and clears the device error word of the
+ * current device: HILL_ERR_TIMEOUT if a bounded wait expired, HILL_ERR_DEVICE
+ * if a device-side argument check fired, HILL_ERR_CUDA if the synchronisation
+ * itself failed, else HILL_OK. */
+hill_status hill_sync_status(void* stream);
+
+/* Static, human-readable name of a status. */
+const char* hill_status_string(hill_status status);
+
+/* Number of kernels this library has launched (or recorded into a CUDA graph
+ * under stream capture) in this process so far, over all devices.  Lets a
+ * caller count the kernels one call or one captured graph contains. */
+uint64_t hill_kernel_launches(void);
+
+/* ABI version of this header (major * 100 + minor). */
+int32_t hill_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HILL_H_ */

@@ -1,0 +1,339 @@
+// api.cu -- the C ABI of libhill (include/hill.h): argument validation,
+// workspace layout and the launch sequence of each call.
+#include <atomic>
+#include <mutex>
+
+#include "../../include/hill.h"
+#include "hill_internal.h"
+
+namespace hill {
+
+// Device error word of this library (reported by hill_sync_status).
+__device__ unsigned int g_error_word = 0;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+constexpr int kMaxDevices = 64;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+struct DeviceInfo {
+  int sms = 0;
+  unsigned* err = nullptr;
+};
+
+std::mutex g_mu;
+DeviceInfo g_dev[kMaxDevices];
+std::atomic<uint64_t> g_launches{0};
+
+cudaError_t counted(cudaError_t e, int kernels) {
+  if (e == cudaSuccess) g_launches.fetch_add((uint64_t)kernels, std::memory_order_relaxed);
+  return e;
+}
+
+// Per-device constants: SM count and the device address of the error word.
+cudaError_t device_info(DeviceInfo* out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_mu);
+  DeviceInfo& d = g_dev[dev];
+  if (d.sms == 0) {
+    int sms = 0;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_error_word);
+    if (e != cudaSuccess) return e;
+    d.err = static_cast<unsigned*>(p);
+    d.sms = sms;
+  }
+  *out = d;
+  return cudaSuccess;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool stride_ok(int64_t s) { return s >= 0 && (s % 8) == 0; }
+
+hill_status check_desc(const hill_desc* d) {
+  if (!d) return HILL_ERR_INVALID_ARG;
+  if (d->batch < 0 || d->num_q_heads <= 0 || d->num_kv_heads <= 0 || d->capacity < 0 || d->head_dim <= 0)
+    return HILL_ERR_INVALID_ARG;
+  if (d->num_q_heads % d->num_kv_heads) return HILL_ERR_INVALID_ARG;
+  if (d->dtype != HILL_F16 && d->dtype != HILL_BF16) return HILL_ERR_INVALID_ARG;
+  if (!stride_ok(d->q_sb) || !stride_ok(d->q_sh) || !stride_ok(d->k_sb) || !stride_ok(d->k_sh) ||
+      !stride_ok(d->k_sn) || !stride_ok(d->v_sb) || !stride_ok(d->v_sh) || !stride_ok(d->v_sn))
+    return HILL_ERR_INVALID_ARG;
+  if (d->head_dim != kHeadDim) return HILL_ERR_UNSUPPORTED;
+  const int G = d->num_q_heads / d->num_kv_heads;
+  if (G != 1 && G != 2 && G != 4 && G != 8) return HILL_ERR_UNSUPPORTED;
+  if (d->batch > score_max_batch()) return HILL_ERR_UNSUPPORTED;
+  if (d->num_kv_heads > score_max_kv_heads(G)) return HILL_ERR_UNSUPPORTED;
+  // the selection keeps a sequence's keys on chip across at most 8 CTAs
+  if (select_smem_bytes(d->capacity, select_cluster_size(d->capacity)) > 220 * 1024)
+    return HILL_ERR_UNSUPPORTED;
+  return HILL_OK;
+}
+
+struct Layout {
+  size_t scores, logits, partials, attn_part, total;
+  int score_grid, splits, per_split;
+};
+
+int score_grid_for(const hill_desc* d, int sms) {
+  const int T = score_tile_tokens();
+  const long long items = (long long)d->batch * ((d->capacity + T - 1) / T);
+  long long g = sms;
+  if (items < g) g = items;
+  return g < 1 ? 1 : (int)g;
+}
+
+void attn_split(const hill_desc* d, int max_k, int sms, int* splits, int* per_split) {
+  const long long units = (long long)d->batch * d->num_kv_heads;
+  long long want = units > 0 ? (4LL * sms + units - 1) / units : 1;
+  long long most = (max_k + 31) / 32;
+  if (want > most) want = most;
+  if (want < 1) want = 1;
+  int per = (int)((max_k + want - 1) / want);
+  if (per < 1) per = 1;
+  *per_split = per;
+  *splits = max_k > 0 ? (max_k + per - 1) / per : 1;
+}
+
+Layout layout_for(const hill_desc* d, int mode, int max_k, int sms) {
+  Layout L{};
+  const size_t B = d->batch, H = d->num_q_heads, cap = d->capacity;
+  L.score_grid = score_grid_for(d, sms);
+  attn_split(d, max_k < 0 ? 0 : max_k, sms, &L.splits, &L.per_split);
+  size_t off = 0;
+  L.scores = off;
+  off += align_up(B * cap * sizeof(float));
+  L.logits = off;
+  if (mode == HILL_SCORE_ATTN) off += align_up(B * H * cap * sizeof(float));
+  L.partials = off;
+  if (mode == HILL_SCORE_ATTN) off += align_up(B * (size_t)L.score_grid * H * sizeof(float2));
+  L.attn_part = off;
+  if (L.splits > 1) off += align_up(B * H * (size_t)L.splits * (2 + kHeadDim) * sizeof(float));
+  L.total = off + kAlign;  // room to align the caller's base pointer
+  return L;
+}
+
+unsigned char* ws_base(void* ws) {
+  uintptr_t p = reinterpret_cast<uintptr_t>(ws);
+  return reinterpret_cast<unsigned char*>((p + kAlign - 1) & ~(uintptr_t)(kAlign - 1));
+}
+
+hill_status from_cuda(cudaError_t e) { return e == cudaSuccess ? HILL_OK : HILL_ERR_CUDA; }
+
+hill_status run_score(const hill_desc* d, const void* q, const void* k, const int32_t* lens, int mode,
+                      float* scores, float* accum, unsigned char* base, const Layout& L,
+                      const DeviceInfo& di, cudaStream_t st) {
+  if (d->batch == 0 || d->capacity == 0) return HILL_OK;
+  const int G = d->num_q_heads / d->num_kv_heads;
+  ScoreArgs a{};
+  a.q = q;
+  a.k = k;
+  a.lens = lens;
+  a.B = d->batch;
+  a.H = d->num_q_heads;
+  a.Hkv = d->num_kv_heads;
+  a.cap = d->capacity;
+  a.q_sb = d->q_sb;
+  a.q_sh = d->q_sh;
+  a.k_sb = d->k_sb;
+  a.k_sh = d->k_sh;
+  a.k_sn = d->k_sn;
+  a.nslot = L.score_grid;
+  a.err = di.err;
+  const bool raw = mode == HILL_SCORE_RAW;
+  if (raw) {
+    a.scores = scores;
+    a.accum = accum;
+  } else {
+    a.logits = reinterpret_cast<float*>(base + L.logits);
+    a.partials = reinterpret_cast<float2*>(base + L.partials);
+  }
+  hill_status s = from_cuda(counted(launch_score(a, d->dtype, G, raw, L.score_grid, st), 1));
+  if (s != HILL_OK || raw) return s;
+  FinalizeArgs f{};
+  f.logits = a.logits;
+  f.partials = a.partials;
+  f.lens = lens;
+  f.B = d->batch;
+  f.H = d->num_q_heads;
+  f.cap = d->capacity;
+  f.nslot = L.score_grid;
+  f.scores = scores;
+  f.accum = accum;
+  return from_cuda(counted(launch_attn_finalize(f, st), 1));
+}
+
+hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens, const int32_t* k,
+                       int max_k, int32_t* idx, int32_t* count, const DeviceInfo& di, cudaStream_t st) {
+  if (d->batch == 0) return HILL_OK;
+  SelectArgs a{};
+  a.key = key;
+  a.lens = lens;
+  a.k = k;
+  a.B = d->batch;
+  a.cap = d->capacity;
+  a.max_k = max_k;
+  a.idx = idx;
+  a.count = count;
+  a.err = di.err;
+  return from_cuda(counted(launch_select(a, st), 1));
+}
+
+hill_status run_attn(const hill_desc* d, const void* q, const void* k, const void* v, const int32_t* idx,
+                     const int32_t* count, int max_k, float* out, unsigned char* base, const Layout& L,
+                     const DeviceInfo& di, cudaStream_t st) {
+  if (d->batch == 0) return HILL_OK;
+  AttnArgs a{};
+  a.q = q;
+  a.k = k;
+  a.v = v;
+  a.idx = idx;
+  a.count = count;
+  a.B = d->batch;
+  a.H = d->num_q_heads;
+  a.Hkv = d->num_kv_heads;
+  a.cap = d->capacity;
+  a.max_k = max_k;
+  a.q_sb = d->q_sb;
+  a.q_sh = d->q_sh;
+  a.k_sb = d->k_sb;
+  a.k_sh = d->k_sh;
+  a.k_sn = d->k_sn;
+  a.v_sb = d->v_sb;
+  a.v_sh = d->v_sh;
+  a.v_sn = d->v_sn;
+  a.out = out;
+  a.part = reinterpret_cast<float*>(base + L.attn_part);
+  a.splits = L.splits;
+  a.per_split = L.per_split;
+  a.err = di.err;
+  return from_cuda(counted(launch_sparse_attn(a, d->dtype, d->num_q_heads / d->num_kv_heads, st),
+                           L.splits > 1 ? 2 : 1));
+}
+
+}  // namespace
+}  // namespace hill
+
+using namespace hill;
+
+extern "C" {
+
+int32_t hill_abi_version(void) { return 100; }
+
+uint64_t hill_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
+
+const char* hill_status_string(hill_status s) {
+  switch (s) {
+    case HILL_OK: return "HILL_OK";
+    case HILL_ERR_INVALID_ARG: return "HILL_ERR_INVALID_ARG";
+    case HILL_ERR_UNSUPPORTED: return "HILL_ERR_UNSUPPORTED";
+    case HILL_ERR_WORKSPACE: return "HILL_ERR_WORKSPACE";
+    case HILL_ERR_CUDA: return "HILL_ERR_CUDA";
+    case HILL_ERR_TIMEOUT: return "HILL_ERR_TIMEOUT";
+    case HILL_ERR_DEVICE: return "HILL_ERR_DEVICE";
+  }
+  return "HILL_ERR_UNKNOWN";
+}
+
+size_t hill_workspace_bytes(const hill_desc* desc, hill_score_mode mode, int32_t max_k) {
+  if (check_desc(desc) != HILL_OK) return 0;
+  if (mode != HILL_SCORE_ATTN && mode != HILL_SCORE_RAW) return 0;
+  if (max_k < 0) return 0;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return 0;
+  return layout_for(desc, mode, max_k, di.sms).total;
+}
+
+hill_status hill_score(const hill_desc* desc, const void* q, const void* k_cache, const int32_t* lens,
+                       hill_score_mode mode, float* scores, float* accum, void* ws, size_t ws_bytes,
+                       void* stream) {
+  hill_status s = check_desc(desc);
+  if (s != HILL_OK) return s;
+  if (mode != HILL_SCORE_ATTN && mode != HILL_SCORE_RAW) return HILL_ERR_INVALID_ARG;
+  if (!q || !k_cache || !lens || !scores) return HILL_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k_cache)) return HILL_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  const Layout L = layout_for(desc, mode, 0, di.sms);
+  if (!ws || ws_bytes < L.total) return HILL_ERR_WORKSPACE;
+  return run_score(desc, q, k_cache, lens, mode, scores, accum, ws_base(ws), L, di,
+                   static_cast<cudaStream_t>(stream));
+}
+
+hill_status hill_topk_select(const hill_desc* desc, const float* scores, const int32_t* lens, const int32_t* k,
+                             int32_t max_k, int32_t* idx, int32_t* count, void* ws, size_t ws_bytes,
+                             void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  hill_status s = check_desc(desc);
+  if (s != HILL_OK) return s;
+  if (max_k < 0 || !scores || !lens || !k || !count || (max_k > 0 && !idx)) return HILL_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  return run_select(desc, scores, lens, k, max_k, idx, count, di, static_cast<cudaStream_t>(stream));
+}
+
+hill_status hill_gather_sparse_attn(const hill_desc* desc, const void* q, const void* k_cache,
+                                    const void* v_cache, const int32_t* idx, const int32_t* count,
+                                    int32_t max_k, float* out, void* ws, size_t ws_bytes, void* stream) {
+  hill_status s = check_desc(desc);
+  if (s != HILL_OK) return s;
+  if (max_k < 0 || !q || !k_cache || !v_cache || !count || !out || (max_k > 0 && !idx))
+    return HILL_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache)) return HILL_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  const Layout L = layout_for(desc, HILL_SCORE_RAW, max_k, di.sms);
+  if (L.splits > 1 && (!ws || ws_bytes < L.total)) return HILL_ERR_WORKSPACE;
+  return run_attn(desc, q, k_cache, v_cache, idx, count, max_k, out, ws ? ws_base(ws) : nullptr, L, di,
+                  static_cast<cudaStream_t>(stream));
+}
+
+hill_status hill_evict_step(const hill_desc* desc, const void* q, const void* k_cache, const void* v_cache,
+                            const int32_t* lens, const int32_t* k, int32_t max_k, hill_score_mode mode,
+                            float* accum, float* scores, int32_t* idx, int32_t* count, float* out, void* ws,
+                            size_t ws_bytes, void* stream) {
+  hill_status s = check_desc(desc);
+  if (s != HILL_OK) return s;
+  if (mode != HILL_SCORE_ATTN && mode != HILL_SCORE_RAW) return HILL_ERR_INVALID_ARG;
+  if (max_k < 0 || !q || !k_cache || !lens || !k || !count || (max_k > 0 && !idx)) return HILL_ERR_INVALID_ARG;
+  if (out && !v_cache) return HILL_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k_cache) || (out && !aligned16(v_cache))) return HILL_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  const Layout L = layout_for(desc, mode, max_k, di.sms);
+  if (!ws || ws_bytes < L.total) return HILL_ERR_WORKSPACE;
+  unsigned char* base = ws_base(ws);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  float* s_out = scores ? scores : (accum ? nullptr : reinterpret_cast<float*>(base + L.scores));
+  s = run_score(desc, q, k_cache, lens, mode, s_out, accum, base, L, di, st);
+  if (s != HILL_OK) return s;
+  const float* key = accum ? accum : s_out;
+  s = run_select(desc, key, lens, k, max_k, idx, count, di, st);
+  if (s != HILL_OK || !out) return s;
+  return run_attn(desc, q, k_cache, v_cache, idx, count, max_k, out, base, L, di, st);
+}
+
+hill_status hill_sync_status(void* stream) {
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return HILL_ERR_CUDA;
+  unsigned w = 0;
+  if (cudaMemcpy(&w, di.err, sizeof(w), cudaMemcpyDeviceToHost) != cudaSuccess) return HILL_ERR_CUDA;
+  if (w) {
+    const unsigned zero = 0;
+    if (cudaMemcpy(di.err, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess) return HILL_ERR_CUDA;
+  }
+  if (w & kErrTimeout) return HILL_ERR_TIMEOUT;
+  if (w & kErrDevArg) return HILL_ERR_DEVICE;
+  return HILL_OK;
+}
+
+}  // extern "C"

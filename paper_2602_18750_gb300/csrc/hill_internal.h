@@ -1,0 +1,94 @@
+// hill_internal.h -- argument blocks and launchers shared between the API
+// translation unit (api.cu) and the kernel translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "hill_common.cuh"
+
+namespace hill {
+
+struct ScoreArgs {
+  const void* q;
+  const void* k;
+  const int32_t* lens;
+  int B, H, Hkv, cap;
+  int64_t q_sb, q_sh, k_sb, k_sh, k_sn;
+  float* scores;      // RAW: per-token sums, may be NULL when accum is given
+  float* accum;       // RAW: running importance (+=), may be NULL
+  float* logits;      // ATTN: [B][H][cap]
+  float2* partials;   // ATTN: [B][nslot][H] (max, sum exp)
+  int nslot;          // = grid size of the launch
+  unsigned* err;
+};
+
+struct FinalizeArgs {
+  const float* logits;
+  const float2* partials;
+  const int32_t* lens;
+  int B, H, cap, nslot;
+  float* scores;      // may be NULL when accum is given
+  float* accum;       // may be NULL
+};
+
+struct SelectArgs {
+  const float* key;   // [B][cap]
+  const int32_t* lens;
+  const int32_t* k;
+  int B, cap, max_k;
+  int chunk;          // filled by the launcher
+  int32_t* idx;
+  int32_t* count;
+  unsigned* err;
+};
+
+struct AttnArgs {
+  const void* q;
+  const void* k;
+  const void* v;
+  const int32_t* idx;
+  const int32_t* count;
+  int B, H, Hkv, cap, max_k;
+  int64_t q_sb, q_sh, k_sb, k_sh, k_sn, v_sb, v_sh, v_sn;
+  float* out;         // [B][H][d]
+  float* part;        // [B*H][splits][2 + d] when splits > 1
+  int splits, per_split;
+  unsigned* err;
+};
+
+// Raise a kernel's dynamic shared-memory limit to `bytes` on the current
+// device if it is not there yet; `cache` (64 entries, one per device) records
+// what was set, so that steady-state launches -- including ones under stream
+// capture -- make no attribute calls.
+inline cudaError_t ensure_smem_attr(const void* func, int bytes, int* cache) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (bytes > cache[dev]) {
+    e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return e;
+    cache[dev] = bytes;
+  }
+  return cudaSuccess;
+}
+
+// score.cu
+size_t score_smem_bytes(int G);
+int score_tile_tokens();
+int score_max_batch();
+int score_max_kv_heads(int G);
+cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, int grid, cudaStream_t st);
+cudaError_t launch_attn_finalize(const FinalizeArgs& a, cudaStream_t st);
+
+// select.cu
+int select_cluster_size(int cap);
+size_t select_smem_bytes(int cap, int C);
+cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
+
+// attn.cu
+cudaError_t launch_sparse_attn(const AttnArgs& a, int dtype, int G, cudaStream_t st);
+
+}  // namespace hill
