@@ -32,6 +32,7 @@ constexpr int kSW = 2;                      // stages per consumer warp
 constexpr int kStages = kNC * kSW;
 constexpr int kThreads = (kNC + 1) * 32;
 constexpr int kMaxBatchSmem = 2048;         // sequences held in the tile prefix table
+constexpr int kTstartInts = kMaxBatchSmem + 4;  // B + 1 entries, padded to keep 16-byte alignment
 constexpr int kRunSlots = 64;               // running (m, l) slots per warp (Hkv/kNC * G)
 
 template <int G>
@@ -59,7 +60,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(ScoreArgs a) {
   uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
   uint64_t* empty_bar = full_bar + kStages;
   int* tstart = reinterpret_cast<int*>(empty_bar + kStages);            // [B+1]
-  float* red = reinterpret_cast<float*>(tstart + kMaxBatchSmem + 1);    // [2][kNC][kT]
+  float* red = reinterpret_cast<float*>(tstart + kTstartInts);          // [2][kNC][kT]
   float2* run = reinterpret_cast<float2*>(red + 2 * kNC * kT);          // [kNC][kRunSlots]
 
   const int warp = threadIdx.x >> 5;
@@ -352,7 +353,7 @@ cudaError_t launch_score_g(const ScoreArgs& a, int G, int grid, cudaStream_t st)
 
 size_t score_smem_bytes(int G) {
   const size_t stage = (size_t)kT * kRowBytes + (size_t)G * kRowBytes;
-  return kStages * stage + 2 * kStages * sizeof(uint64_t) + (kMaxBatchSmem + 1) * sizeof(int) +
+  return kStages * stage + 2 * kStages * sizeof(uint64_t) + kTstartInts * sizeof(int) +
          2 * kNC * kT * sizeof(float) + kNC * kRunSlots * sizeof(float2);
 }
 

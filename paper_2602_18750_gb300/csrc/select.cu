@@ -196,7 +196,11 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
       take = eq_rank < remaining;
       ++eq_rank;
     }
-    if (take) out[pos++] = j_lo + i;
+    if (take) {
+      if (pos < (uint32_t)kk) out[pos] = j_lo + i;
+      else raise_error(a.err, kErrDevArg);   // cannot happen: more picks than the budget
+      ++pos;
+    }
   }
 }
 
