@@ -90,23 +90,18 @@ int score_grid_for(const hill_desc* d, int sms) {
   return g < 1 ? 1 : (int)g;
 }
 
-void attn_split(const hill_desc* d, int max_k, int sms, int* splits, int* per_split) {
-  const long long units = (long long)d->batch * d->num_kv_heads;
-  long long want = units > 0 ? (4LL * sms + units - 1) / units : 1;
-  long long most = (max_k + 31) / 32;
-  if (want > most) want = most;
-  if (want < 1) want = 1;
-  int per = (int)((max_k + want - 1) / want);
-  if (per < 1) per = 1;
-  *per_split = per;
-  *splits = max_k > 0 ? (max_k + per - 1) / per : 1;
+// The attention grid covers max_k in chunks of attn_chunk_tokens() entries.
+void attn_split(int max_k, int* splits, int* per_split) {
+  const int c = attn_chunk_tokens();
+  *per_split = c;
+  *splits = max_k > c ? (max_k + c - 1) / c : 1;
 }
 
 Layout layout_for(const hill_desc* d, int mode, int max_k, int sms) {
   Layout L{};
   const size_t B = d->batch, H = d->num_q_heads, cap = d->capacity;
   L.score_grid = score_grid_for(d, sms);
-  attn_split(d, max_k < 0 ? 0 : max_k, sms, &L.splits, &L.per_split);
+  attn_split(max_k < 0 ? 0 : max_k, &L.splits, &L.per_split);
   size_t off = 0;
   L.scores = off;
   off += align_up(B * cap * sizeof(float));

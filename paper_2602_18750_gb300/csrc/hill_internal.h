@@ -89,6 +89,7 @@ size_t select_smem_bytes(int cap, int C);
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
 
 // attn.cu
+int attn_chunk_tokens();
 cudaError_t launch_sparse_attn(const AttnArgs& a, int dtype, int G, cudaStream_t st);
 
 }  // namespace hill

@@ -1,15 +1,17 @@
 // select.cu -- per-sequence top-k selection (Sec. 3.1 top-alpha retention;
 // Sec. 4.2: the global top-alpha after merging every score source).
 //
-// One thread-block cluster of C CTAs per sequence.  Each CTA holds a
-// contiguous chunk of the sequence's scores in shared memory as 32-bit
-// order-preserving keys; the cluster finds the exact k-th largest key with a
-// three-pass MSD radix select (11 + 11 + 10 bits).  Every pass histograms the
-// keys that match the digits fixed so far; CTA r merges bins [r*W, (r+1)*W)
-// of all CTAs' histograms through distributed shared memory, and the CTA
-// holding the crossing bin broadcasts the next digit.  This is the GPU form
-// of the paper's merge of chunked <position, score> blocks (Sec. 4.2): the
-// chunks stay on chip and only bin counts cross between CTAs.
+// A sequence's scores are held on chip as 32-bit order-preserving keys, by
+// one CTA when they fit (up to kChunkMax keys), otherwise by a thread-block
+// cluster of C CTAs, each holding a contiguous chunk.  The exact k-th largest
+// key is found by an MSD radix select with digits of 11, 11 and 10 bits.  In
+// each pass every CTA histograms the keys that match the digits fixed so
+// far; CTA r merges bins [r*W, (r+1)*W) of all CTAs' histograms through
+// distributed shared memory and publishes its bin total; every CTA then finds
+// the crossing bin itself by reading the owner's merged bins.  A pass ends
+// the search early when the crossing bin is taken whole.  This is the GPU
+// form of the paper's merge of chunked <position, score> blocks (Sec. 4.2):
+// the chunks stay on chip and only bin counts cross between CTAs.
 //
 // Ties at the boundary go to the lowest token index: with tau the k-th key
 // and r_eq the number of keys equal to tau that must be taken, a token is
@@ -25,49 +27,66 @@ namespace cg = cooperative_groups;
 namespace hill {
 namespace {
 
-constexpr int kSelThreads = 512;
+constexpr int kSelThreads = 1024;
 constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kBins = 2048;
-constexpr int kMaxCluster = 16;
+constexpr int kMaxCluster = 8;
+constexpr int kChunkMax = 16384;   // keys per CTA before the cluster grows
 
 // Exclusive prefix sum over the block (thread order); *total gets the sum.
+// wsum needs kSelWarps + 1 entries.
 __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* wsum, uint32_t* total) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   uint32_t x = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+    const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
     if (lane >= o) x += y;
   }
   __syncthreads();  // wsum may still be read by a previous scan
   if (lane == 31) wsum[warp] = x;
   __syncthreads();
-  uint32_t base = 0, all = 0;
+  if (warp == 0) {
+    const uint32_t t = lane < kSelWarps ? wsum[lane] : 0u;
+    uint32_t u = t;
 #pragma unroll
-  for (int w = 0; w < kSelWarps; ++w) {
-    const uint32_t t = wsum[w];
-    base += (w < warp) ? t : 0u;
-    all += t;
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, u, o);
+      if (lane >= o) u += y;
+    }
+    if (lane < kSelWarps) wsum[lane] = u - t;
+    if (lane == 31) wsum[kSelWarps] = u;
   }
-  *total = all;
-  return base + x - v;
+  __syncthreads();
+  *total = wsum[kSelWarps];
+  return wsum[warp] + x - v;
 }
 
+template <bool CL>
 __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) {
+  int C = 1, r = 0;
   cg::cluster_group cluster = cg::this_cluster();
-  const int C = (int)cluster.num_blocks();
-  const int r = (int)cluster.block_rank();
+  if (CL) {
+    C = (int)cluster.num_blocks();
+    r = (int)cluster.block_rank();
+  }
+  auto csync = [&]() {
+    if (CL) cluster.sync(); else __syncthreads();
+  };
+  auto remote = [&](uint32_t* p, int c) -> uint32_t* {
+    return CL ? cluster.map_shared_rank(p, c) : p;
+  };
   const int b = blockIdx.y;
   const int tid = threadIdx.x;
 
   extern __shared__ uint32_t sm[];
   uint32_t* keys = sm;                   // [chunk]
   uint32_t* hist = keys + a.chunk;       // [kBins]
-  uint32_t* merged = hist + kBins;       // [kBins]  (only [0, kBins / C) used)
-  __shared__ uint32_t wsum[kSelWarps];
+  uint32_t* merged = hist + kBins;       // [kBins] (only [0, nb / C) used)
+  __shared__ uint32_t wsum[kSelWarps + 1];
   __shared__ uint32_t tot[kMaxCluster];
   __shared__ uint32_t cgt[kMaxCluster], ceq[kMaxCluster];
-  __shared__ uint32_t bc[2];
+  __shared__ uint32_t bc[3];
 
   int len = a.lens[b];
   len = len < 0 ? 0 : (len > a.cap ? a.cap : len);
@@ -96,6 +115,7 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
 
   uint32_t prefix = 0, pmask = 0;
   uint32_t remaining = (uint32_t)kk;
+  bool take_bucket = false;    // the crossing bucket is taken whole
 #pragma unroll 1
   for (int pass = 0; pass < 3; ++pass) {
     const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
@@ -107,61 +127,71 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
       const uint32_t kv = keys[i];
       if ((kv & pmask) == prefix) atomicAdd(&hist[(kv >> shift) & dmask], 1u);
     }
-    cluster.sync();  // every local histogram is complete
+    csync();  // (A) every local histogram is complete
 
-    const int W = nb / C;
-    const int base = r * W;
-    uint32_t part = 0;
-    for (int i = tid; i < W; i += kSelThreads) {
-      uint32_t s = 0;
-      for (int c = 0; c < C; ++c) s += cluster.map_shared_rank(hist, c)[base + i];
-      merged[i] = s;
-      part += s;
-    }
-    uint32_t mine;
-    (void)block_excl_scan(part, wsum, &mine);
-    if (tid == 0)
-      for (int c = 0; c < C; ++c) cluster.map_shared_rank(tot, c)[r] = mine;
-    cluster.sync();  // totals everywhere; remote histogram reads finished
-
-    // which CTA's bin range holds the remaining-th largest matching key?
+    int W = nb;
     uint32_t above = 0;
     int owner = 0;
-    for (int c = C - 1; c >= 0; --c) {
-      if (above + tot[c] >= remaining) { owner = c; break; }
-      above += tot[c];
-    }
-    if (r == owner) {
-      // positions p = 0.. run over the owned bins from the top down
-      const int per = (W + kSelThreads - 1) / kSelThreads;
-      const int p0 = tid * per;
-      uint32_t s = 0;
-      for (int p = p0; p < min(p0 + per, W); ++p) s += merged[W - 1 - p];
-      uint32_t tall;
-      const uint32_t ex = block_excl_scan(s, wsum, &tall);
-      if (above + ex < remaining && remaining <= above + ex + s) {
-        uint32_t cum = above + ex;
-        for (int p = p0; p < min(p0 + per, W); ++p) {
-          const uint32_t c = merged[W - 1 - p];
-          if (cum + c >= remaining) {
-            const uint32_t digit = (uint32_t)(base + W - 1 - p);
-            for (int q = 0; q < C; ++q) {
-              uint32_t* rb = cluster.map_shared_rank(bc, q);
-              rb[0] = digit;
-              rb[1] = remaining - cum;
-            }
-            break;
-          }
-          cum += c;
+    const uint32_t* om = hist;
+    if (CL) {
+      W = nb / C;
+      const int base = r * W;
+      uint32_t part = 0;
+      for (int i = tid; i < W; i += kSelThreads) {
+        uint32_t s = 0;
+        for (int c = 0; c < C; ++c) s += remote(hist, c)[base + i];
+        merged[i] = s;
+        part += s;
+      }
+      uint32_t mine;
+      (void)block_excl_scan(part, wsum, &mine);
+      if (tid == 0)
+        for (int c = 0; c < C; ++c) remote(tot, c)[r] = mine;
+      csync();  // (B) merged bins and totals published; remote histogram reads done
+      // which CTA's bin range holds the remaining-th largest matching key?
+      for (int c = C - 1; c >= 0; --c) {
+        if (above + tot[c] >= remaining) {
+          owner = c;
+          break;
         }
+        above += tot[c];
+      }
+      om = remote(merged, owner);
+    }
+    // positions p = 0.. run over the owner's bins from the top down
+    const int per = (W + kSelThreads - 1) / kSelThreads;
+    const int p0 = tid * per;
+    const int p1 = min(p0 + per, W);
+    uint32_t s = 0;
+    for (int p = p0; p < p1; ++p) s += om[W - 1 - p];
+    uint32_t tall;
+    const uint32_t ex = block_excl_scan(s, wsum, &tall);
+    if (above + ex < remaining && remaining <= above + ex + s) {
+      uint32_t cum = above + ex;
+      for (int p = p0; p < p1; ++p) {
+        const uint32_t c = om[W - 1 - p];
+        if (cum + c >= remaining) {
+          bc[0] = (uint32_t)(owner * W + W - 1 - p);
+          bc[1] = remaining - cum;
+          bc[2] = c;
+          break;
+        }
+        cum += c;
       }
     }
-    cluster.sync();  // digit broadcast
+    __syncthreads();
     prefix |= bc[0] << shift;
     pmask |= dmask << shift;
     remaining = bc[1];
+    if (remaining == bc[2]) {
+      take_bucket = true;
+      break;
+    }
   }
-  const uint32_t tau = prefix;   // the k-th largest key; `remaining` ties at tau are taken
+  // Selection rule: take_bucket -> key >= prefix (every key of the crossing
+  // bucket and above); otherwise tau = prefix is the k-th key itself and
+  // `remaining` of the keys equal to tau are taken, lowest index first.
+  const uint32_t tau = prefix;
 
   // ---------------------------------------------------------------- compaction
   const int per = (n + kSelThreads - 1) / kSelThreads;
@@ -169,32 +199,42 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
   uint32_t my_gt = 0, my_eq = 0;
   for (int i = i0; i < i1; ++i) {
     const uint32_t kv = keys[i];
-    my_gt += kv > tau;
-    my_eq += kv == tau;
+    if (take_bucket) {
+      my_gt += kv >= tau;
+    } else {
+      my_gt += kv > tau;
+      my_eq += kv == tau;
+    }
   }
   uint32_t tgt, teq;
   const uint32_t gt_ex = block_excl_scan(my_gt, wsum, &tgt);
   const uint32_t eq_ex = block_excl_scan(my_eq, wsum, &teq);
-  if (tid == 0)
-    for (int c = 0; c < C; ++c) {
-      cluster.map_shared_rank(cgt, c)[r] = tgt;
-      cluster.map_shared_rank(ceq, c)[r] = teq;
-    }
-  cluster.sync();
+  if (CL) {
+    if (tid == 0)
+      for (int c = 0; c < C; ++c) {
+        remote(cgt, c)[r] = tgt;
+        remote(ceq, c)[r] = teq;
+      }
+    csync();
+  }
   uint32_t gt_before = 0, eq_before = 0;
   for (int c = 0; c < r; ++c) {
     gt_before += cgt[c];
     eq_before += ceq[c];
   }
-  // ties taken before this thread's segment, and the output position of its first pick
-  uint32_t eq_rank = eq_before + eq_ex;
+  uint32_t eq_rank = eq_before + eq_ex;   // ties before this thread's segment
   uint32_t pos = gt_before + gt_ex + min(eq_rank, remaining);
   for (int i = i0; i < i1; ++i) {
     const uint32_t kv = keys[i];
-    bool take = kv > tau;
-    if (kv == tau) {
-      take = eq_rank < remaining;
-      ++eq_rank;
+    bool take;
+    if (take_bucket) {
+      take = kv >= tau;
+    } else {
+      take = kv > tau;
+      if (kv == tau) {
+        take = eq_rank < remaining;
+        ++eq_rank;
+      }
     }
     if (take) {
       if (pos < (uint32_t)kk) out[pos] = j_lo + i;
@@ -207,9 +247,8 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
 }  // namespace
 
 int select_cluster_size(int cap) {
-  int need = (cap + 4095) / 4096;
   int C = 1;
-  while (C < need && C < 8) C <<= 1;
+  while (C < kMaxCluster && (cap + C - 1) / C > kChunkMax) C <<= 1;
   return C;
 }
 
@@ -223,22 +262,30 @@ cudaError_t launch_select(const SelectArgs& a0, cudaStream_t st) {
   const int C = select_cluster_size(a.cap);
   a.chunk = (a.cap + C - 1) / C;
   const size_t smem = select_smem_bytes(a.cap, C);
-  static int cache[64] = {0};
-  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(hill_select_kernel), (int)smem, cache);
-  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(C, a.B, 1);
   cfg.blockDim = dim3(kSelThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = C;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, hill_select_kernel, a);
+  cudaError_t e;
+  if (C == 1) {
+    static int cache[64] = {0};
+    e = ensure_smem_attr(reinterpret_cast<const void*>(hill_select_kernel<false>), (int)smem, cache);
+    if (e != cudaSuccess) return e;
+    e = cudaLaunchKernelEx(&cfg, hill_select_kernel<false>, a);
+  } else {
+    static int cache[64] = {0};
+    e = ensure_smem_attr(reinterpret_cast<const void*>(hill_select_kernel<true>), (int)smem, cache);
+    if (e != cudaSuccess) return e;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = C;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, hill_select_kernel<true>, a);
+  }
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
