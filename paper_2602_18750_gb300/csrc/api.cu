@@ -1,5 +1,8 @@
 // api.cu -- the C ABI of libhill (include/hill.h): argument validation,
 // workspace layout and the launch sequence of each call.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
 #include <atomic>
 #include <mutex>
 
@@ -54,6 +57,62 @@ cudaError_t device_info(DeviceInfo* out) {
   return cudaSuccess;
 }
 
+// cuTensorMapEncodeTiled from the driver, resolved through the runtime (no
+// link-time dependency on libcuda).
+PFN_cuTensorMapEncodeTiled_v12000 encode_tiled() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// Tiled tensor map of the key cache for hill_score_kernel: dimension 0 is the
+// head dimension (contiguous, box 64 = 128 bytes, 128-byte swizzle); the
+// token, KV-head and sequence dimensions follow in increasing stride order
+// (so token-major caches work too), with a box of 32 tokens.
+hill_status make_kmap(const hill_desc* d, const void* k, ScoreArgs* a) {
+  auto fn = encode_tiled();
+  if (!fn) return HILL_ERR_CUDA;
+  struct Dim {
+    int64_t n, stride;
+    int which;  // 0 token, 1 head, 2 sequence
+  } v[3] = {{d->capacity, d->k_sn, 0}, {d->num_kv_heads, d->k_sh, 1}, {d->batch, d->k_sb, 2}};
+  std::stable_sort(v, v + 3, [](const Dim& x, const Dim& y) { return x.stride < y.stride; });
+  cuuint64_t gdim[4] = {(cuuint64_t)kHeadDim, 1, 1, 1};
+  cuuint64_t gstr[3];
+  cuuint32_t box[4] = {64, 1, 1, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  for (int i = 0; i < 3; ++i) {
+    gdim[i + 1] = (cuuint64_t)std::max<int64_t>(v[i].n, 1);
+    // a dimension of extent 1 may carry any stride; keep it valid and ordered
+    int64_t st = v[i].stride;
+    if (v[i].n <= 1) st = std::max<int64_t>(st, i ? (int64_t)gstr[i - 1] / 2 : kHeadDim);
+    gstr[i] = (cuuint64_t)(st * 2);
+    if (v[i].which == 0) {
+      box[i + 1] = 32;
+      a->kdim_tok = i + 1;
+    } else if (v[i].which == 1) {
+      a->kdim_head = i + 1;
+    } else {
+      a->kdim_seq = i + 1;
+    }
+  }
+  for (int i = 0; i < 3; ++i)
+    if (gstr[i] == 0 || (gstr[i] & 15)) return HILL_ERR_UNSUPPORTED;
+  const CUtensorMapDataType dt =
+      d->dtype == HILL_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+  CUresult r = fn(&a->kmap, dt, 4, const_cast<void*>(k), gdim, gstr, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? HILL_OK : HILL_ERR_UNSUPPORTED;
+}
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 bool stride_ok(int64_t s) { return s >= 0 && (s % 8) == 0; }
 
@@ -69,7 +128,7 @@ hill_status check_desc(const hill_desc* d) {
   if (d->head_dim != kHeadDim) return HILL_ERR_UNSUPPORTED;
   const int G = d->num_q_heads / d->num_kv_heads;
   if (G != 1 && G != 2 && G != 4 && G != 8) return HILL_ERR_UNSUPPORTED;
-  if (d->batch > score_max_batch()) return HILL_ERR_UNSUPPORTED;
+  if (d->batch > score_max_batch() || d->batch > attn_max_batch()) return HILL_ERR_UNSUPPORTED;
   if (d->num_kv_heads > score_max_kv_heads(G)) return HILL_ERR_UNSUPPORTED;
   // the selection keeps a sequence's keys on chip across at most 8 CTAs
   if (select_smem_bytes(d->capacity, select_cluster_size(d->capacity)) > 220 * 1024)
@@ -79,7 +138,7 @@ hill_status check_desc(const hill_desc* d) {
 
 struct Layout {
   size_t scores, logits, partials, attn_part, total;
-  int score_grid, splits, per_split;
+  int score_grid, attn_grid, splits;
 };
 
 int score_grid_for(const hill_desc* d, int sms) {
@@ -90,18 +149,12 @@ int score_grid_for(const hill_desc* d, int sms) {
   return g < 1 ? 1 : (int)g;
 }
 
-// The attention grid covers max_k in chunks of attn_chunk_tokens() entries.
-void attn_split(int max_k, int* splits, int* per_split) {
-  const int c = attn_chunk_tokens();
-  *per_split = c;
-  *splits = max_k > c ? (max_k + c - 1) / c : 1;
-}
-
 Layout layout_for(const hill_desc* d, int mode, int max_k, int sms) {
   Layout L{};
   const size_t B = d->batch, H = d->num_q_heads, cap = d->capacity;
   L.score_grid = score_grid_for(d, sms);
-  attn_split(max_k < 0 ? 0 : max_k, &L.splits, &L.per_split);
+  L.attn_grid = sms;
+  L.splits = attn_max_segments(max_k < 0 ? 0 : max_k);
   size_t off = 0;
   L.scores = off;
   off += align_up(B * cap * sizeof(float));
@@ -110,7 +163,7 @@ Layout layout_for(const hill_desc* d, int mode, int max_k, int sms) {
   L.partials = off;
   if (mode == HILL_SCORE_ATTN) off += align_up(B * (size_t)L.score_grid * H * sizeof(float2));
   L.attn_part = off;
-  if (L.splits > 1) off += align_up(B * H * (size_t)L.splits * (2 + kHeadDim) * sizeof(float));
+  off += align_up(B * H * (size_t)L.splits * (2 + kHeadDim) * sizeof(float));
   L.total = off + kAlign;  // room to align the caller's base pointer
   return L;
 }
@@ -142,6 +195,8 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   a.k_sn = d->k_sn;
   a.nslot = L.score_grid;
   a.err = di.err;
+  hill_status ms = make_kmap(d, k, &a);
+  if (ms != HILL_OK) return ms;
   const bool raw = mode == HILL_SCORE_RAW;
   if (raw) {
     a.scores = scores;
@@ -207,10 +262,8 @@ hill_status run_attn(const hill_desc* d, const void* q, const void* k, const voi
   a.out = out;
   a.part = reinterpret_cast<float*>(base + L.attn_part);
   a.splits = L.splits;
-  a.per_split = L.per_split;
   a.err = di.err;
-  return from_cuda(counted(launch_sparse_attn(a, d->dtype, d->num_q_heads / d->num_kv_heads, st),
-                           L.splits > 1 ? 2 : 1));
+  return from_cuda(counted(launch_sparse_attn(a, d->dtype, d->num_q_heads / d->num_kv_heads, L.attn_grid, st), 2));
 }
 
 }  // namespace
@@ -286,8 +339,8 @@ hill_status hill_gather_sparse_attn(const hill_desc* desc, const void* q, const 
   DeviceInfo di;
   if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
   const Layout L = layout_for(desc, HILL_SCORE_RAW, max_k, di.sms);
-  if (L.splits > 1 && (!ws || ws_bytes < L.total)) return HILL_ERR_WORKSPACE;
-  return run_attn(desc, q, k_cache, v_cache, idx, count, max_k, out, ws ? ws_base(ws) : nullptr, L, di,
+  if (!ws || ws_bytes < L.total) return HILL_ERR_WORKSPACE;
+  return run_attn(desc, q, k_cache, v_cache, idx, count, max_k, out, ws_base(ws), L, di,
                   static_cast<cudaStream_t>(stream));
 }
 

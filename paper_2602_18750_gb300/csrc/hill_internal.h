@@ -2,6 +2,7 @@
 // translation unit (api.cu) and the kernel translation units.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -11,6 +12,8 @@
 namespace hill {
 
 struct ScoreArgs {
+  CUtensorMap kmap;   // K cache: 4-D tiled map, 128-byte swizzle, box = 64 dims x kT tokens
+  int kdim_tok, kdim_head, kdim_seq;   // which tensor-map dimension holds token, KV head, sequence
   const void* q;
   const void* k;
   const int32_t* lens;
@@ -53,8 +56,8 @@ struct AttnArgs {
   int B, H, Hkv, cap, max_k;
   int64_t q_sb, q_sh, k_sb, k_sh, k_sn, v_sb, v_sh, v_sn;
   float* out;         // [B][H][d]
-  float* part;        // [B*H][splits][2 + d] when splits > 1
-  int splits, per_split;
+  float* part;        // [B*H][splits][2 + d] partials of split (b, g) pairs
+  int splits;         // partial slots per (b, h)
   unsigned* err;
 };
 
@@ -75,9 +78,39 @@ inline cudaError_t ensure_smem_attr(const void* func, int bytes, int* cache) {
   return cudaSuccess;
 }
 
+// Launch `kern` as a programmatic dependent of the preceding kernel in the
+// stream (its prologue may overlap that kernel's tail; the kernel itself
+// calls pdl_wait() before touching data the predecessor produced), with an
+// optional cluster shape.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       int cluster_x, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  int n = 1;
+  if (cluster_x > 0) {
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = cluster_x;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    n = 2;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kern, args...);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 // score.cu
 size_t score_smem_bytes(int G);
 int score_tile_tokens();
+int score_warps();
 int score_max_batch();
 int score_max_kv_heads(int G);
 cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, int grid, cudaStream_t st);
@@ -89,7 +122,9 @@ size_t select_smem_bytes(int cap, int C);
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
 
 // attn.cu
-int attn_chunk_tokens();
-cudaError_t launch_sparse_attn(const AttnArgs& a, int dtype, int G, cudaStream_t st);
+int attn_batch_tokens();
+int attn_max_batch();
+int attn_max_segments(int max_k);
+cudaError_t launch_sparse_attn(const AttnArgs& a, int dtype, int G, int grid, cudaStream_t st);
 
 }  // namespace hill

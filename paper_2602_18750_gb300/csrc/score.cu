@@ -2,27 +2,27 @@
 // the ATTN-mode normalisation (Sec. 4.1 column sum of softmax weights).
 //
 // hill_score_kernel: persistent CTAs of kNW warps.  A work item is a tile of
-// kT consecutive tokens of one sequence; the KV heads g of an item are dealt
-// to the warps (g mod kNW).  Every warp streams its own (item, g) sequence
-// through a private ring of kSW shared-memory stages: lane 0 issues one bulk
-// TMA copy of the tile's kT key rows (kT x 256 B, or kT row copies when the
-// rows are strided) plus the G query rows of the head group, completing on
-// the stage's mbarrier; the warp copies a landed stage into registers, hands
-// the slot straight back to the copy engine for the stage kSW ahead, and
-// computes.  Each lane owns 16 bytes of a row (a half-warp covers one 256-B
-// row), keeps fp32 partial sums for 16 rows and finishes them with a
-// 15-shuffle transposed reduction, after which lane l holds token
-// 2*(l%16) + l/16 of the tile.
+// kT = 32 consecutive tokens of one sequence; the KV heads g of an item are
+// dealt to the warps (g mod kNW).  Every warp streams its own (item, g)
+// sequence through a private ring of kSW shared-memory stages: lane 0 issues
+// two tiled TMA loads (dims 0-63 and 64-127 of the tile's 32 key rows, 128-
+// byte swizzle) plus a bulk copy of the G query rows of the head group, all
+// completing on the stage's mbarrier.  The warp moves a landed tile into
+// registers with ldmatrix (conflict-free thanks to the swizzle), hands the
+// slot back to the copy engine for the stage kSW ahead, and computes the
+// [32 tokens x 128] . [128 x G heads] product with 16 mma.sync m16n8k16
+// (fp32 accumulation; the G query heads fill the N = 8 columns, so one
+// instruction stream serves MHA and GQA alike).
 //
 //   RAW : the per-token sum over heads is reduced across the warps in shared
 //         memory at the end of each item (fixed order) and written to scores
-//         (and added to accum).  The RAW importance is linear in q, so the G
-//         query heads of a group are summed first (one dot product per row).
-//   ATTN: every logit z = q.K/sqrt(d) is written to a [B][H][cap] buffer and
-//         each lane keeps an online (max, sum exp) of its tokens per head;
-//         when the CTA leaves a sequence the warp merges them and writes one
-//         partial per (sequence, head, CTA).  hill_attn_finalize_kernel
-//         combines the partials and forms s[b,j] = sum_h exp(z - m_bh) / L_bh.
+//         (and added to accum).
+//   ATTN: every logit z = q.K/sqrt(d) is written to a [B][H][cap] buffer; per
+//         stage the warp reduces each head's tile (max, sum exp) and merges it
+//         into a running state in shared memory; when the CTA leaves a
+//         sequence the warp writes one partial per (sequence, head, CTA).
+//         hill_attn_finalize_kernel combines the partials and forms
+//         s[b,j] = sum_h exp(z[b,h,j] - m_bh) / L_bh.
 #include "hill_internal.h"
 
 namespace hill {
@@ -34,13 +34,22 @@ constexpr int kNW = 8;                      // warps per CTA
 constexpr int kThreads = kNW * 32;
 constexpr int kMaxBatchSmem = 512;          // sequences held in the per-CTA tables
 constexpr int kTableInts = kMaxBatchSmem + 4;  // B + 1 entries, padded (16-byte alignment)
-constexpr int kMaxRun = 8;                  // (KV heads per warp) x G online-softmax states per lane
+constexpr int kMaxNg = 4;                   // KV heads per warp per item (Hkv <= kNW * kMaxNg)
+constexpr int kBoxBytes = kT * 128;         // one 64-dim half of a tile: 32 swizzled 128-byte rows
+constexpr int kKBytes = 2 * kBoxBytes;
 
 template <int G>
 struct ScoreCfg {
-  static constexpr int kStageBytes = kT * kRowBytes + G * kRowBytes;
+  static constexpr int kSlotBytes = ((kKBytes + G * kRowBytes + 1023) / 1024) * 1024;
   static constexpr int kSW = G <= 4 ? 3 : 2;             // stages per warp
   static constexpr int kStages = kNW * kSW;
+  // shared-memory layout (offsets from a 1024-byte aligned base)
+  static constexpr int kOffBar = kStages * kSlotBytes;
+  static constexpr int kOffTab = kOffBar + kStages * 8;
+  static constexpr int kOffRed = kOffTab + 2 * kTableInts * 4;
+  static constexpr int kOffStat = kOffRed + 2 * kNW * kT * 4;
+  static constexpr int kOffFlag = kOffStat + kNW * kMaxNg * 8 * 8;
+  static constexpr int kBytes = kOffFlag + 16 + 1024;        // + alignment slack
 };
 
 __device__ __forceinline__ int find_seq(const int* tstart, int B, int item) {
@@ -52,29 +61,15 @@ __device__ __forceinline__ int find_seq(const int* tstart, int B, int item) {
   return lo;
 }
 
-// Online (max, sum exp) of one lane's tokens.
-__device__ __forceinline__ void online_push(float& m, float& l, float z) {
-  if (z > m) {
-    l = l * expf(m - z) + 1.f;
-    m = z;
-  } else {
-    l += expf(z - m);
-  }
-}
-
-__device__ __forceinline__ void online_merge_warp(float& m, float& l) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
-    const float l2 = __shfl_xor_sync(0xffffffffu, l, o);
-    const float mx = fmaxf(m, m2);
-    l = (mx == -INFINITY) ? 0.f : l * expf(m - mx) + l2 * expf(m2 - mx);
-    m = mx;
-  }
-}
-
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Merge two (max, sum exp) pairs.
+__device__ __forceinline__ float2 merge_ml(float2 x, float2 y) {
+  const float m = fmaxf(x.x, y.x);
+  if (m == -INFINITY) return make_float2(-INFINITY, 0.f);
+  return make_float2(m, x.y * expf(x.x - m) + y.y * expf(y.x - m));
 }
 
 // Position of a warp in its own stage sequence: item (global tile index) and
@@ -84,32 +79,34 @@ struct Cursor {
 };
 
 template <int DT, int G, bool RAW>
-__global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(ScoreArgs a) {
+__global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_constant__ ScoreArgs a) {
   using Cfg = ScoreCfg<G>;
-  constexpr int kStageBytes = Cfg::kStageBytes;
+  constexpr int kSlotBytes = Cfg::kSlotBytes;
   constexpr int kSW = Cfg::kSW;
   constexpr int kStages = Cfg::kStages;
-  constexpr int kNH = RAW ? 1 : (G < 4 ? G : 4);   // heads per pass over a stage
-  constexpr int kPasses = RAW ? 1 : G / kNH;
-  constexpr int kMaxNg = RAW ? 1 : kMaxRun / G;    // KV heads per warp per item (ATTN)
 
-  extern __shared__ __align__(1024) unsigned char smem[];
-  unsigned char* stage_base = smem;
-  uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
-  int* tstart = reinterpret_cast<int*>(full_bar + kStages);             // [B+1] tile prefix
-  int* slen = tstart + kTableInts;                                      // [B] clamped lengths
-  float* red = reinterpret_cast<float*>(slen + kTableInts);             // [2][kNW][kT]
-  __shared__ int abort_flag;
+  extern __shared__ unsigned char smem_raw[];
+  const uint32_t raw_addr = smem_addr(smem_raw);
+  const uint32_t base_addr = (raw_addr + 1023u) & ~1023u;
+  unsigned char* base = smem_raw + (base_addr - raw_addr);
+  int* tstart = reinterpret_cast<int*>(base + Cfg::kOffTab);          // [B+1] tile prefix
+  int* slen = tstart + kTableInts;                                     // [B] clamped lengths
+  float* red = reinterpret_cast<float*>(base + Cfg::kOffRed);          // [2][kNW][kT]
+  float2* stat = reinterpret_cast<float2*>(base + Cfg::kOffStat);      // [kNW][kMaxNg][8]
+  volatile int* abort_flag = reinterpret_cast<int*>(base + Cfg::kOffFlag);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int B = a.B, H = a.H, Hkv = a.Hkv, cap = a.cap;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) mbar_init(smem_addr(&full_bar[s]), 1);
+    for (int s = 0; s < kStages; ++s) mbar_init(base_addr + Cfg::kOffBar + s * 8, 1);
     fence_barrier_init();
-    abort_flag = 0;
+    *abort_flag = 0;
+    prefetch_tmap(&a.kmap);
   }
+  pdl_wait();
+  pdl_launch_dependents();
   for (int b = threadIdx.x; b < B; b += kThreads) {
     int len = a.lens[b];
     if (len < 0 || len > cap) {
@@ -119,6 +116,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(ScoreArgs a) {
     slen[b] = len;
   }
   __syncthreads();
+  // an item holds every KV head of one tile
   if (threadIdx.x == 0) {
     int acc = 0;
     tstart[0] = 0;
@@ -129,13 +127,12 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(ScoreArgs a) {
   }
   __syncthreads();
   const int n_items = tstart[B];
-  const int ng = (Hkv - warp + kNW - 1) / kNW;   // KV heads of this warp per item
+  const int ng = (Hkv - warp + kNW - 1) / kNW;   // KV heads of this warp per tile
 
   const uint64_t pol = l2_evict_first_policy();
-  const auto* kbase = static_cast<const uint16_t*>(a.k);
   const auto* qbase = static_cast<const uint16_t*>(a.q);
-  const uint32_t stage0 = smem_addr(stage_base) + warp * kSW * kStageBytes;
-  const uint32_t bar0 = smem_addr(&full_bar[warp * kSW]);
+  const uint32_t stage0 = base_addr + warp * kSW * kSlotBytes;
+  const uint32_t bar0 = base_addr + Cfg::kOffBar + warp * kSW * 8;
 
   auto advance = [&](Cursor& c) {
     if (++c.r >= ng) {
@@ -147,26 +144,33 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(ScoreArgs a) {
   auto issue = [&](const Cursor& c, uint32_t no) {
     const int b = find_seq(tstart, B, c.item);
     const int j0 = (c.item - tstart[b]) * kT;
-    const int nv = min(kT, slen[b] - j0);
     const int g = warp + c.r * kNW;
     const uint32_t s = no % kSW;
     const uint32_t fb = bar0 + s * 8;
-    const uint32_t dst = stage0 + s * kStageBytes;
-    mbar_arrive_expect_tx(fb, (uint32_t)(nv + G) * kRowBytes);
-    const uint16_t* ksrc = kbase + (int64_t)b * a.k_sb + (int64_t)g * a.k_sh + (int64_t)j0 * a.k_sn;
-    if (a.k_sn == kHeadDim) {
-      bulk_g2s(dst, ksrc, (uint32_t)nv * kRowBytes, fb, pol);
-    } else {
-      for (int r = 0; r < nv; ++r) bulk_g2s(dst + r * kRowBytes, ksrc + (int64_t)r * a.k_sn, kRowBytes, fb, pol);
-    }
+    const uint32_t dst = stage0 + s * kSlotBytes;
+    mbar_arrive_expect_tx(fb, (uint32_t)(kKBytes + G * kRowBytes));
+    int crd[4] = {0, 0, 0, 0};
+    crd[a.kdim_tok] = j0;
+    crd[a.kdim_head] = g;
+    crd[a.kdim_seq] = b;
+    tma_load_4d(dst, &a.kmap, 0, crd[1], crd[2], crd[3], fb, pol);
+    tma_load_4d(dst + kBoxBytes, &a.kmap, 64, crd[1], crd[2], crd[3], fb, pol);
     const uint16_t* qsrc = qbase + (int64_t)b * a.q_sb + (int64_t)(g * G) * a.q_sh;
-    const uint32_t qdst = dst + kT * kRowBytes;
+    const uint32_t qdst = dst + kKBytes;
     if (a.q_sh == kHeadDim) {
       bulk_g2s(qdst, qsrc, G * kRowBytes, fb);
     } else {
 #pragma unroll
       for (int r = 0; r < G; ++r) bulk_g2s(qdst + r * kRowBytes, qsrc + (int64_t)r * a.q_sh, kRowBytes, fb);
     }
+  };
+
+  // per-warp running (max, sum exp) of each (stage slot r, head) of the current sequence
+  float2* wstat = stat + warp * kMaxNg * 8;
+  auto reset_stat = [&]() {
+    __syncwarp();
+    wstat[lane] = make_float2(-INFINITY, 0.f);   // kMaxNg * 8 == 32 entries
+    __syncwarp();
   };
 
   // prologue: the first kSW stages of this warp
@@ -179,72 +183,82 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(ScoreArgs a) {
     }
   }
 
-  const int l16 = lane & 15;
-  const int half = lane >> 4;
-  const int tok = 2 * l16 + half;          // token (within the tile) this lane ends with
+  // fragment coordinates (mma.sync m16n8k16): C row = token lane/4 (+8),
+  // C columns = heads 2*(lane%4) and 2*(lane%4)+1 of the group
+  const int grp = lane >> 2, tig = lane & 3;
+  const int hA = 2 * tig, hB = 2 * tig + 1;
+  // ldmatrix row address pieces: matrix m = lane/8 covers rows (m&1)*8.., k half m>>1
+  const int lm_row = (lane & 7) + ((lane >> 3) & 1) * 8;
+  const int lm_khalf = lane >> 4;
   uint32_t used = 0;                       // stages consumed
   int item_no = 0;
   bool ok = true;
-
-  float run_m[RAW ? 1 : kMaxRun], run_l[RAW ? 1 : kMaxRun];
   int cur_b = -1, cur_slot = 0;
-  auto reset_run = [&]() {
-#pragma unroll
-    for (int e = 0; e < (RAW ? 1 : kMaxRun); ++e) {
-      run_m[e] = -INFINITY;
-      run_l[e] = 0.f;
-    }
-  };
+  if (!RAW) reset_stat();
+
   auto flush = [&]() {
-    if (RAW) return;
-#pragma unroll
-    for (int r = 0; r < kMaxNg; ++r) {
-      if (r >= ng) break;
-#pragma unroll
-      for (int hl = 0; hl < G; ++hl) {
-        float m = run_m[r * G + hl], l = run_l[r * G + hl];
-        online_merge_warp(m, l);
+    if constexpr (!RAW) {
+      __syncwarp();
+      if (lane < ng * G) {
+        const int r = lane / G, hl = lane % G;
         const int h = (warp + r * kNW) * G + hl;
-        if (lane == 0) a.partials[((int64_t)cur_b * a.nslot + cur_slot) * H + h] = make_float2(m, l);
+        a.partials[((int64_t)cur_b * a.nslot + cur_slot) * H + h] = wstat[r * 8 + hl];
       }
+      __syncwarp();
     }
   };
-  reset_run();
 
   for (int item = blockIdx.x; item < n_items; item += gridDim.x, ++item_no) {
     const int b = find_seq(tstart, B, item);
     const int tile = item - tstart[b];
     const int j0 = tile * kT;
     const int nv = min(kT, slen[b] - j0);
-    const bool valid = tok < nv;
-    float rsum = 0.f;
+    float rs[4] = {0.f, 0.f, 0.f, 0.f};   // RAW: token sums of rows grp, grp+8, 16+grp, 24+grp
 
     if (!RAW && b != cur_b) {
       if (cur_b >= 0) flush();
-      reset_run();
+      reset_stat();
       cur_b = b;
-      cur_slot = tile;   // = item - tstart[b]: this CTA's first item in b
+      cur_slot = tile;   // = item - tstart[b]: this CTA's first item in b (< gridDim.x)
     }
 
 #pragma unroll 1
     for (int r = 0; r < ng && ok; ++r) {
       const int g = warp + r * kNW;
+      const int sr = r;   // running-state slot of this KV head
       const uint32_t s = used % kSW;
       if (!mbar_wait(bar0 + s * 8, (used / kSW) & 1u, a.err)) {
         ok = false;
-        abort_flag = 1;
+        *abort_flag = 1;
         break;
       }
-      const uint32_t sb = stage0 + s * kStageBytes;
-      const uint32_t qb = sb + kT * kRowBytes;
-      // copy the stage into registers, then refill the slot with the stage
-      // kSW ahead while this one is computed
-      uint4 kv[16];
+      const uint32_t sb = stage0 + s * kSlotBytes;
+      const uint32_t qb = sb + kKBytes;
+      // K tile -> A fragments (2 blocks of 16 tokens x 8 blocks of 16 dims)
+      uint32_t af[2][8][4];
 #pragma unroll
-      for (int it = 0; it < 16; ++it) kv[it] = lds128(sb + (2 * it + half) * kRowBytes + l16 * 16);
-      uint4 qv[G];
+      for (int mb = 0; mb < 2; ++mb) {
+        const int t = mb * 16 + lm_row;
 #pragma unroll
-      for (int hh = 0; hh < G; ++hh) qv[hh] = lds128(qb + hh * kRowBytes + l16 * 16);
+        for (int kb = 0; kb < 8; ++kb) {
+          const int chunk = kb * 2 + lm_khalf;          // 16-byte chunk of the 256-byte row
+          const uint32_t addr = sb + (chunk >> 3) * kBoxBytes + t * 128 + (((chunk & 7) ^ (t & 7)) << 4);
+          ldmatrix_x4(addr, af[mb][kb]);
+        }
+      }
+      // q rows -> B fragments (rows n >= G of the 8 columns are zero)
+      uint32_t bf[8][2];
+#pragma unroll
+      for (int kb = 0; kb < 8; ++kb) {
+        if (grp < G) {
+          const uint32_t qa = qb + grp * kRowBytes + (kb * 16 + tig * 2) * 2;
+          bf[kb][0] = lds32(qa);
+          bf[kb][1] = lds32(qa + 16);
+        } else {
+          bf[kb][0] = 0u;
+          bf[kb][1] = 0u;
+        }
+      }
       ++used;
       __syncwarp();
       if (pc.item < n_items) {
@@ -256,53 +270,75 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(ScoreArgs a) {
         advance(pc);
       }
 
+      float acc[2][4];
 #pragma unroll
-      for (int pass = 0; pass < kPasses; ++pass) {
-        float qf[kNH][8];
-        if (RAW) {
+      for (int mb = 0; mb < 2; ++mb)
 #pragma unroll
-          for (int e = 0; e < 8; ++e) qf[0][e] = 0.f;
+        for (int e = 0; e < 4; ++e) acc[mb][e] = 0.f;
 #pragma unroll
-          for (int hh = 0; hh < G; ++hh) {
-            float t[8];
-            to_float8<DT>(qv[hh], t);
+      for (int kb = 0; kb < 8; ++kb)
 #pragma unroll
-            for (int e = 0; e < 8; ++e) qf[0][e] += t[e];
-          }
-        } else {
+        for (int mb = 0; mb < 2; ++mb) mma_16816<DT>(acc[mb], af[mb][kb], bf[kb][0], bf[kb][1]);
+
+      // acc[mb][0|1] = token mb*16 + grp, heads hA|hB; acc[mb][2|3] = token mb*16 + grp + 8
+      if (RAW) {
 #pragma unroll
-          for (int hh = 0; hh < kNH; ++hh) to_float8<DT>(qv[pass * kNH + hh], qf[hh]);
+        for (int u = 0; u < 4; ++u) {
+          const int mb = u >> 1, e = (u & 1) * 2;
+          float v = (hA < G ? acc[mb][e] : 0.f) + (hB < G ? acc[mb][e + 1] : 0.f);
+          v += __shfl_xor_sync(0xffffffffu, v, 1);
+          v += __shfl_xor_sync(0xffffffffu, v, 2);
+          rs[u] += v * kInvSqrtD;
         }
-        float acc[kNH][16];
+      } else {
+        float zA[4], zB[4];
+        bool tv[4];
 #pragma unroll
-        for (int it = 0; it < 16; ++it) {
-          float kf[8];
-          to_float8<DT>(kv[it], kf);
-#pragma unroll
-          for (int hh = 0; hh < kNH; ++hh) {
-            float sum = 0.f;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) sum = fmaf(qf[hh][e], kf[e], sum);
-            acc[hh][it] = sum;
-          }
+        for (int u = 0; u < 4; ++u) {
+          const int mb = u >> 1, e = (u & 1) * 2;
+          zA[u] = acc[mb][e] * kInvSqrtD;
+          zB[u] = acc[mb][e + 1] * kInvSqrtD;
+          tv[u] = (mb * 16 + grp + (u & 1) * 8) < nv;
         }
+        float* lg = a.logits + ((int64_t)b * H + g * G) * cap + j0;
 #pragma unroll
-        for (int hh = 0; hh < kNH; ++hh) {
-          const float z = half_transpose_reduce(acc[hh], lane) * kInvSqrtD;
-          if (RAW) {
-            rsum += z;
-          } else {
-            const int hl = pass * kNH + hh;            // head within the group
-            const int h = g * G + hl;
-            if (valid) {
-              a.logits[((int64_t)b * H + h) * cap + j0 + tok] = z;
-              // r is warp-uniform; select the register slot with a static index
-#pragma unroll
-              for (int rr = 0; rr < kMaxNg; ++rr)
-                if (rr == r) online_push(run_m[rr * G + hl], run_l[rr * G + hl], z);
-            }
+        for (int u = 0; u < 4; ++u) {
+          const int t = (u >> 1) * 16 + grp + (u & 1) * 8;
+          if (tv[u]) {
+            if (hA < G) lg[(int64_t)hA * cap + t] = zA[u];
+            if (hB < G) lg[(int64_t)hB * cap + t] = zB[u];
           }
         }
+        // tile (max, sum exp) of heads hA and hB over the 8 lanes of this column pair
+        float mA = -INFINITY, mB = -INFINITY;
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (tv[u]) {
+            mA = fmaxf(mA, zA[u]);
+            mB = fmaxf(mB, zB[u]);
+          }
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {
+          mA = fmaxf(mA, __shfl_xor_sync(0xffffffffu, mA, o));
+          mB = fmaxf(mB, __shfl_xor_sync(0xffffffffu, mB, o));
+        }
+        float lA = 0.f, lB = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (tv[u]) {
+            lA += expf(zA[u] - mA);
+            lB += expf(zB[u] - mB);
+          }
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {
+          lA += __shfl_xor_sync(0xffffffffu, lA, o);
+          lB += __shfl_xor_sync(0xffffffffu, lB, o);
+        }
+        if (lane < 4) {
+          if (hA < G) wstat[sr * 8 + hA] = merge_ml(wstat[sr * 8 + hA], make_float2(mA, lA));
+          if (hB < G) wstat[sr * 8 + hB] = merge_ml(wstat[sr * 8 + hB], make_float2(mB, lB));
+        }
+        __syncwarp();
       }
     }
     if (RAW) {
@@ -310,14 +346,17 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(ScoreArgs a) {
       // whose wait timed out still reaches the barrier, and all warps then
       // leave together
       float* rb = red + (item_no & 1) * kNW * kT;
-      rb[warp * kT + tok] = rsum;
+      if (tig == 0) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) rb[warp * kT + (u >> 1) * 16 + grp + (u & 1) * 8] = rs[u];
+      }
       named_sync(1, kThreads);
-      if (abort_flag) break;
-      if (warp == (item_no % kNW) && valid) {
+      if (*abort_flag) break;
+      if (warp == (item_no % kNW) && lane < nv) {
         float sum = 0.f;
 #pragma unroll
-        for (int w = 0; w < kNW; ++w) sum += rb[w * kT + tok];
-        const int64_t o = (int64_t)b * cap + j0 + tok;
+        for (int w = 0; w < kNW; ++w) sum += rb[w * kT + lane];
+        const int64_t o = (int64_t)b * cap + j0 + lane;
         if (a.scores) a.scores[o] = sum;
         if (a.accum) a.accum[o] += sum;
       }
@@ -347,13 +386,15 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   extern __shared__ float fsm[];
   float* mh = fsm;            // [H]
   float* il = fsm + a.H;      // [H]
+  pdl_wait();
+  pdl_launch_dependents();
   const int b = blockIdx.y;
   int len = a.lens[b];
   len = len < 0 ? 0 : (len > a.cap ? a.cap : len);
   const int jb = blockIdx.x * kFinChunk;
   if (jb >= len) return;
-  const int tiles = (len + kT - 1) / kT;
-  const int ns = min(tiles, a.nslot);
+  const int items = (len + kT - 1) / kT;
+  const int ns = min(items, a.nslot);
   const float2* pb = a.partials + (int64_t)b * a.nslot * a.H;
   const int sub = threadIdx.x % kFinPartThreads;
   for (int h = threadIdx.x / kFinPartThreads; h < a.H; h += kFinThreads / kFinPartThreads) {
@@ -412,8 +453,7 @@ cudaError_t launch_score_t(const ScoreArgs& a, int grid, cudaStream_t st) {
   static int cache[64] = {0};
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), (int)smem, cache);
   if (e != cudaSuccess) return e;
-  kern<<<grid, kThreads, smem, st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(grid), dim3(kThreads), smem, st, 0, a);
 }
 
 template <int DT, bool RAW>
@@ -429,9 +469,7 @@ cudaError_t launch_score_g(const ScoreArgs& a, int G, int grid, cudaStream_t st)
 
 template <int G>
 size_t smem_for() {
-  using Cfg = ScoreCfg<G>;
-  return (size_t)Cfg::kStages * Cfg::kStageBytes + Cfg::kStages * sizeof(uint64_t) +
-         2 * kTableInts * sizeof(int) + 2 * kNW * kT * sizeof(float);
+  return (size_t)ScoreCfg<G>::kBytes;
 }
 
 }  // namespace
@@ -446,8 +484,12 @@ size_t score_smem_bytes(int G) {
 }
 
 int score_tile_tokens() { return kT; }
+int score_warps() { return kNW; }
 int score_max_batch() { return kMaxBatchSmem; }
-int score_max_kv_heads(int G) { return (kMaxRun / G) * kNW; }
+int score_max_kv_heads(int G) {
+  (void)G;
+  return kMaxNg * kNW;
+}
 
 cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, int grid, cudaStream_t st) {
   if (dtype == 0) return raw ? launch_score_g<0, true>(a, G, grid, st) : launch_score_g<0, false>(a, G, grid, st);
@@ -456,8 +498,7 @@ cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, int gri
 
 cudaError_t launch_attn_finalize(const FinalizeArgs& a, cudaStream_t st) {
   dim3 grid((a.cap + kFinChunk - 1) / kFinChunk, a.B);
-  hill_attn_finalize_kernel<<<grid, kFinThreads, 2 * a.H * sizeof(float), st>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(hill_attn_finalize_kernel, grid, dim3(kFinThreads), 2 * a.H * sizeof(float), st, 0, a);
 }
 
 }  // namespace hill

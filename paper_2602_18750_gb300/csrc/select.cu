@@ -27,7 +27,7 @@ namespace cg = cooperative_groups;
 namespace hill {
 namespace {
 
-constexpr int kSelThreads = 1024;
+constexpr int kSelThreads = 512;
 constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kBins = 2048;
 constexpr int kMaxCluster = 8;
@@ -78,6 +78,8 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
   };
   const int b = blockIdx.y;
   const int tid = threadIdx.x;
+  pdl_wait();
+  pdl_launch_dependents();
 
   extern __shared__ uint32_t sm[];
   uint32_t* keys = sm;                   // [chunk]
@@ -262,32 +264,17 @@ cudaError_t launch_select(const SelectArgs& a0, cudaStream_t st) {
   const int C = select_cluster_size(a.cap);
   a.chunk = (a.cap + C - 1) / C;
   const size_t smem = select_smem_bytes(a.cap, C);
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(C, a.B, 1);
-  cfg.blockDim = dim3(kSelThreads, 1, 1);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = st;
-  cudaError_t e;
+  const dim3 grid(C, a.B, 1), block(kSelThreads, 1, 1);
   if (C == 1) {
     static int cache[64] = {0};
-    e = ensure_smem_attr(reinterpret_cast<const void*>(hill_select_kernel<false>), (int)smem, cache);
+    cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(hill_select_kernel<false>), (int)smem, cache);
     if (e != cudaSuccess) return e;
-    e = cudaLaunchKernelEx(&cfg, hill_select_kernel<false>, a);
-  } else {
-    static int cache[64] = {0};
-    e = ensure_smem_attr(reinterpret_cast<const void*>(hill_select_kernel<true>), (int)smem, cache);
-    if (e != cudaSuccess) return e;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = C;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, hill_select_kernel<true>, a);
+    return launch_pdl(hill_select_kernel<false>, grid, block, smem, st, 0, a);
   }
+  static int cache[64] = {0};
+  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(hill_select_kernel<true>), (int)smem, cache);
   if (e != cudaSuccess) return e;
-  return cudaGetLastError();
+  return launch_pdl(hill_select_kernel<true>, grid, block, smem, st, C, a);
 }
 
 }  // namespace hill
