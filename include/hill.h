@@ -7,7 +7,7 @@
  * (Sec. 4.1 column-sum of attention weights, or the raw inner product of
  * Sec. 4.4), optionally add them to a running per-token importance, select
  * the top-k tokens per sequence (Sec. 3.1, Sec. 4.2), and run the decode
- * attention over the selected tokens only (Sec. 3.1, step 6).
+ * attention over the selected tokens only (Sec. 4.1, workflow step 6).
  *
  * Conventions shared by every call
  * --------------------------------
@@ -103,7 +103,7 @@ hill_status hill_topk_select(const hill_desc* desc, const float* scores, const i
                              const int32_t* k, int32_t max_k, int32_t* idx, int32_t* count,
                              void* ws, size_t ws_bytes, void* stream);
 
-/* Decode attention over the selected tokens only (Sec. 3.1 step 6; Eq. 1
+/* Decode attention over the selected tokens only (Sec. 4.1, workflow step 6; Eq. 1
  * restricted to the selected set, softmax renormalised over it):
  *   out[b][h][:] = sum_{t<count[b]} p_t V[b][g(h)][idx[b][t]][:],
  *   p = softmax_t(q_h . K[b][g(h)][idx[b][t]] / sqrt(d)).

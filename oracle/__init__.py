@@ -14,7 +14,7 @@ arrays into it.  Each wrapper names the part of the paper it follows:
                           Sec. 4.4 (raw inner product, RAW)
 * :func:`accumulate`   -- running importance across decode steps (Sec. 4.2)
 * :func:`topk`         -- top-alpha selection (Sec. 3.1, Sec. 4.2)
-* :func:`sparse_attn`  -- attention over the selected KV only (Sec. 3.1 step 6)
+* :func:`sparse_attn`  -- attention over the selected KV only (Sec. 4.1, workflow step 6)
 * :func:`evict_step`   -- the five steps in order
 
 Pins: tests/test_oracle_pins.py checks every function against library

@@ -222,7 +222,7 @@ int oracle_topk(int B, int cap, const int32_t* lens, const double* key,
 
 /*
  * Step 5 -- attention of the current query over the selected tokens only
- * (Sec. 3.1 step 6: only the critical KV is brought to the GPU for the
+ * (Sec. 4.1, workflow step 6: only the critical KV is brought to the GPU for the
  * attention; Eq. 1 restricted to the selected set, the softmax renormalised
  * over that set):
  *   o[b,h,:] = sum_{t<count[b]} p_t V[b,g,idx_t,:],

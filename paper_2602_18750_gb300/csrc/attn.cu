@@ -1,4 +1,4 @@
-// attn.cu -- decode attention over the selected tokens only (Sec. 3.1 step 6:
+// attn.cu -- decode attention over the selected tokens only (Sec. 4.1, workflow step 6:
 // only the critical KV reaches the attention; Eq. 1 restricted to the set).
 //
 // Gather + split-K flash decode on persistent CTAs.  The work is a list of
