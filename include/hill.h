@@ -134,6 +134,34 @@ hill_status hill_sync_status(void* stream);
 /* Static, human-readable name of a status. */
 const char* hill_status_string(hill_status status);
 
+/* Largest scratch, in bytes, that hill_score_noalloc may use: 16 MiB. */
+#define HILL_SCORE_NOALLOC_MAX_SCRATCH (16u << 20)
+
+/* hill_score for callers that cannot allocate device memory.  (The paper
+ * has no counterpart; this is a deployment convenience.)  Some callers have
+ * no way to obtain a workspace: a plug-in running inside a host application
+ * that owns the whole device-memory budget and forbids its own cudaMalloc, a
+ * latency-critical decode loop where an allocation could block or fail at an
+ * unpredictable moment, or a binding from a language without a CUDA
+ * allocator.  This entry point takes the same arguments as hill_score minus
+ * the workspace and computes exactly what hill_score computes; its scratch is
+ * a fixed HILL_SCORE_NOALLOC_MAX_SCRATCH-byte array built into the library,
+ * which every GPU that loads the library holds until the process exits.
+ *  - It allocates nothing: no cudaMalloc, cudaFree or allocating library call.
+ *  - The first call on each device looks up that array's device address
+ *    (cudaGetSymbolAddress, no allocation); make that first call on a device
+ *    before any stream capture.
+ *  - A call needing more scratch than the array holds returns
+ *    HILL_ERR_WORKSPACE without launching anything.  ATTN mode needs about
+ *    4*B*cap*(H + 1) + 8*B*H*SMs bytes; RAW about 4*B*cap.
+ *  - All calls share the array, and it keeps whatever the last call left;
+ *    no entry of it needs to start at zero (a call reads only what it wrote).
+ *    Calls that overlap on the GPU (two streams, or two host threads without
+ *    ordering) race on it: order them on one stream. */
+hill_status hill_score_noalloc(const hill_desc* desc, const void* q, const void* k_cache,
+                               const int32_t* lens, hill_score_mode mode, float* scores,
+                               float* accum, void* stream);
+
 /* Number of kernels this library has launched (or recorded into a CUDA graph
  * under stream capture) in this process so far, over all devices.  Lets a
  * caller count the kernels one call or one captured graph contains. */

@@ -385,3 +385,55 @@ hill_status hill_sync_status(void* stream) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// hill_score_noalloc: hill_score with its scratch in a fixed device array, for
+// callers that cannot allocate device memory (see include/hill.h).
+namespace hill {
+namespace {
+
+// The scratch of hill_score_noalloc.  Every GPU that loads this library
+// holds these bytes until the process exits; all calls share them.
+static __device__ __align__(256) unsigned char g_score_scratch[HILL_SCORE_NOALLOC_MAX_SCRATCH];
+
+void* g_scratch_dev[kMaxDevices];
+
+// Device address of g_score_scratch on the current device, looked up once per
+// device (host code cannot use the symbol itself as a device address).
+cudaError_t score_scratch_address(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_mu);
+  if (!g_scratch_dev[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_score_scratch);
+    if (e != cudaSuccess) return e;
+    g_scratch_dev[dev] = p;
+  }
+  *out = g_scratch_dev[dev];
+  return cudaSuccess;
+}
+
+}  // namespace
+}  // namespace hill
+
+extern "C" hill_status hill_score_noalloc(const hill_desc* desc, const void* q, const void* k_cache,
+                                          const int32_t* lens, hill_score_mode mode, float* scores,
+                                          float* accum, void* stream) {
+  hill_status s = check_desc(desc);
+  if (s != HILL_OK) return s;
+  if (mode != HILL_SCORE_ATTN && mode != HILL_SCORE_RAW) return HILL_ERR_INVALID_ARG;
+  if (!q || !k_cache || !lens || !scores) return HILL_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k_cache)) return HILL_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  const Layout L = layout_for(desc, mode, 0, di.sms);
+  // the array is already 256-byte aligned: the alignment slack is not needed
+  if (L.total - kAlign > (size_t)HILL_SCORE_NOALLOC_MAX_SCRATCH) return HILL_ERR_WORKSPACE;
+  void* scratch = nullptr;
+  if (score_scratch_address(&scratch) != cudaSuccess) return HILL_ERR_CUDA;
+  return run_score(desc, q, k_cache, lens, mode, scores, accum, static_cast<unsigned char*>(scratch), L, di,
+                   static_cast<cudaStream_t>(stream));
+}

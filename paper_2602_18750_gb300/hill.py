@@ -70,6 +70,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_topk_select.argtypes = [D, P, P, P, I32, P, P, P, SZ, P]
     lib.hill_gather_sparse_attn.argtypes = [D, P, P, P, P, P, I32, P, P, SZ, P]
     lib.hill_evict_step.argtypes = [D, P, P, P, P, P, I32, I32, P, P, P, P, P, P, SZ, P]
+    lib.hill_score_noalloc.argtypes = [D, P, P, P, I32, P, P, P]
+    lib.hill_score_noalloc.restype = I32
     lib.hill_sync_status.argtypes = [P]
     lib.hill_status_string.argtypes = [I32]
     lib.hill_status_string.restype = ctypes.c_char_p
@@ -150,6 +152,13 @@ def hill_score(desc, q, k_cache, lens, mode, scores, accum=None, ws=None, stream
     wp, wn = _ws(ws)
     _check(load().hill_score(ctypes.byref(desc), _ptr(q), _ptr(k_cache), _ptr(lens), int(mode),
                              _ptr(scores), _ptr(accum), wp, wn, _stream(stream)), "hill_score")
+
+
+def hill_score_noalloc(desc, q, k_cache, lens, mode, scores, accum=None, stream=None) -> None:
+    """hill_score without a workspace: scratch lives in a fixed array inside
+    the library (for callers that cannot allocate device memory)."""
+    _check(load().hill_score_noalloc(ctypes.byref(desc), _ptr(q), _ptr(k_cache), _ptr(lens), int(mode),
+                                     _ptr(scores), _ptr(accum), _stream(stream)), "hill_score_noalloc")
 
 
 def hill_topk_select(desc, scores, lens, k, max_k, idx, count, ws=None, stream=None) -> None:
