@@ -317,6 +317,46 @@ def run_ours(args):
     k_gbs = world * tokens * k_bytes_per_token / (ms / 1e3) / 1e9
     gpu_launches = sum(launches[t] for t in order)
 
+    # ---------------- evaluation + selection only (no attention): the same steps
+    # with out = NULL, one graph per decode step, timed like the main region
+    def issue_eval(t, st):
+        for l in range(L):
+            r = l % lres
+            hill.hill_evict_step(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], max_k, mode,
+                                 accum[r] if accum is not None else None, scores[l], idx[l], count[l],
+                                 None, ws, st)
+
+    eval_graphs = []
+    for t in range(S):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            issue_eval(t, stream)
+        eval_graphs.append(g)
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            eval_graphs[i % S].replay()
+    barrier(dev)
+    torch.cuda.synchronize(dev)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for t in order:
+            eval_graphs[t].replay()
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(dev)
+    ms_eval = max_over_ranks(e0.elapsed_time(e1), dev)
+    hill.hill_sync_status(stream)
+    eval_gbs = tokens * k_bytes_per_token / (ms_eval / 1e3) / 1e9
+    peak, peak_kind = measured_peaks()
+    eval_select = {
+        "what": "hill_evict_step without attention (score + aggregate + select), all layers",
+        "us_per_layer": round(ms_eval * 1e3 / (len(order) * L), 2),
+        "tokens_per_s": round(world * tokens / (ms_eval / 1e3), 1),
+        "k_stream_gbs": round(eval_gbs, 1),
+        "k_stream_frac_of_measured_hbm": round(eval_gbs / peak, 4),
+        "k_stream_frac_of_8tbs": round(eval_gbs / 8000.0, 4),
+    }
+
     # ---------------- scoring stage alone, per launch (roofline of the dominant kernels)
     t_s = S - 1
     lens_s = w.lens_at(t_s)
@@ -370,6 +410,7 @@ def run_ours(args):
             "k_stream_frac_of_measured_hbm": round(k_gbs / world / peak, 4),
             "k_stream_frac_of_8tbs": round(k_gbs / world / 8000.0, 4),
             "eval_step_us_per_layer": round(step_us_per_layer, 2),
+            "eval_select": eval_select,
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": gpu_launches,
             "clocks": clock_info, "generate_s": round(t_gen, 1),
         }
