@@ -5,19 +5,23 @@
 // batches: (sequence b, KV head g, batch bi of 32 consecutive entries of
 // b's index list), ordered b, g, bi.  Every warp of the grid owns one
 // contiguous segment of that list and streams it through two shared-memory
-// slots: each batch's 32 K rows, 32 V rows (tokens idx[b][32*bi + i]) and the
-// G query rows of the head group are gathered with 16-byte asynchronous
-// copies (one cp.async group per batch, a half-warp per 256-byte row); the
-// indices of the batch after next are loaded while the current one computes.
-// (Per-row bulk TMA copies were measured slower here: at 256 bytes each the
-// copy engine's per-request cost, not DRAM, bounds the gather.)  Lanes then own
-// 16 bytes of a row (a half-warp covers one row), partial dots for 16 rows
-// finish with the transposed reduction, an online softmax keeps (max, sum,
-// o) per query head across the batches of one (b, g), and the V rows are
-// accumulated with the weights shuffled back to the lanes that read them.
-// When a warp's segment holds all batches of a (b, g) it writes the output;
-// otherwise it writes a partial (max, sum, o) that hill_attn_combine_kernel
-// merges.
+// slots.  A batch's 32 K rows and 32 V rows (tokens idx[b][32*bi + i]) and
+// the G query rows of the head group are gathered with 16-byte asynchronous
+// copies (one cp.async group per batch, a half-warp per 256-byte row) into
+// an XOR-swizzled layout that ldmatrix reads without bank conflicts; rows of
+// absent tokens are zero-filled.  The index entries of the batch after next
+// are loaded while the current one computes and are checked only when that
+// batch is issued.  (TMA alternatives were measured slower on the same
+// layout: 256-byte bulk copies per row are bound by the copy engine's
+// request rate, and tile::gather4 loads reached about 85 % of the cp.async
+// throughput; neither depends on how scattered the rows are.)
+// Both products run on mma.sync m16n8k16 with fp32 accumulation: S^T =
+// q . K^T (the G query heads are the rows, K rows read with ldmatrix), an
+// online softmax per head across the batches of one (b, g), and O += P . V
+// with V read by transposed ldmatrix; the weights P enter the tensor cores
+// as a 16-bit high part plus its 16-bit residual.  When a warp's segment
+// holds all batches of a (b, g) it writes the output; otherwise it writes a
+// partial (max, sum, o) that hill_attn_combine_kernel merges.
 #include "hill_internal.h"
 
 namespace hill {
@@ -28,10 +32,13 @@ constexpr int kAThreads = kAW * 32;
 constexpr int kBatch = 32;                           // selected entries per batch
 constexpr int kMaxBatchAttn = 512;                   // sequences in the per-CTA table
 
+constexpr int kHalfBytes = kBatch * 128;             // 32 rows x 64 dims, swizzled
+
 template <int G>
 struct AttnCfg {
-  static constexpr int kSlotBytes = 2 * kBatch * kRowBytes + G * kRowBytes;   // K, V, q
-  static constexpr int kSmem = kAW * 2 * kSlotBytes;
+  // K dims 0-63 | K dims 64-127 | V dims 0-63 | V dims 64-127 | q rows
+  static constexpr int kSlotBytes = ((4 * kHalfBytes + G * kRowBytes + 1023) / 1024) * 1024;
+  static constexpr int kSmem = kAW * 2 * kSlotBytes + 1024;   // + alignment slack
 };
 
 // Batch list bookkeeping shared by the attention and combine kernels.
@@ -66,19 +73,22 @@ __device__ __forceinline__ void warp_segment(int total, int nwarps, int w, int& 
 }
 
 template <int DT, int G>
-__global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(AttnArgs a) {
+__global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __grid_constant__ AttnArgs a) {
   using Cfg = AttnCfg<G>;
-  extern __shared__ __align__(128) unsigned char asmem[];
+  extern __shared__ unsigned char asmem[];
   __shared__ int s_bstart[kMaxBatchAttn + 1];
   __shared__ int s_nbat[kMaxBatchAttn];
+  __shared__ int s_cnt[kMaxBatchAttn];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int l16 = lane & 15, half = lane >> 4;
-  const int tok = 2 * l16 + half;
   pdl_wait();
   pdl_launch_dependents();
 
-  for (int b = threadIdx.x; b < a.B; b += kAThreads) s_nbat[b] = (clamp_count(a, b) + kBatch - 1) / kBatch;
+  for (int b = threadIdx.x; b < a.B; b += kAThreads) {
+    const int n = clamp_count(a, b);
+    s_cnt[b] = n;
+    s_nbat[b] = (n + kBatch - 1) / kBatch;
+  }
   __syncthreads();
   if (threadIdx.x == 0) {
     int acc = 0;
@@ -95,45 +105,52 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(AttnArgs
   warp_segment(total, gridDim.x * kAW, blockIdx.x * kAW + warp, t0, t1);
   if (t0 >= t1) return;
 
-  const uint32_t slot0 = smem_addr(asmem) + warp * 2 * Cfg::kSlotBytes;
+  const uint32_t base_addr = (smem_addr(asmem) + 1023u) & ~1023u;
+  const uint32_t slot0 = base_addr + warp * 2 * Cfg::kSlotBytes;
   const auto* qbase = static_cast<const uint16_t*>(a.q);
-  const auto* kbase = static_cast<const uint16_t*>(a.k);
-  const auto* vbase = static_cast<const uint16_t*>(a.v);
 
-  // token index of this lane for batch t (-1 if none)
+  // raw index entry of this lane for batch t (-1 past the count).  Nothing
+  // here depends on the loaded value, so the load stays in flight until the
+  // batch is issued one iteration later, where it is checked.
   auto load_idx = [&](int t) -> int {
     int b, g, bi;
     tab.decode(t, b, g, bi);
     const int e = bi * kBatch + lane;
-    int j = e < clamp_count(a, b) ? a.idx[(int64_t)b * a.max_k + e] : -1;
-    if (j >= a.cap || (j < 0 && e < clamp_count(a, b))) {
-      raise_error(a.err, kErrDevArg);
-      j = -1;
-    }
-    return j;
+    return e < s_cnt[b] ? a.idx[(int64_t)b * a.max_k + e] : -1;
   };
   // gather batch t into slot s: row r of the batch is token jj of lane r
-  // (-1: nothing to copy); one cp.async group per batch
+  // (-1: none, zero-filled).  A half-warp copies one 256-byte row; chunk c
+  // (16 bytes) of row r goes to 128-byte line r of half c / 8 at position
+  // (c % 8) ^ (r % 8), so the ldmatrix reads below are conflict-free.
   auto issue = [&](int t, int s, int jj) {
     int b, g, bi;
     tab.decode(t, b, g, bi);
+    if (bi * kBatch + lane < s_cnt[b] && (jj < 0 || jj >= a.cap)) {
+      raise_error(a.err, kErrDevArg);   // a listed entry outside [0, cap): skipped
+      jj = -1;
+    }
     const unsigned vm = __ballot_sync(0xffffffffu, jj >= 0);
     const uint32_t sk = slot0 + s * Cfg::kSlotBytes;
-    const uint16_t* kr = kbase + (int64_t)b * a.k_sb + (int64_t)g * a.k_sh + l16 * 8;
-    const uint16_t* vr = vbase + (int64_t)b * a.v_sb + (int64_t)g * a.v_sh + l16 * 8;
-#pragma unroll
-    for (int it = 0; it < 16; ++it) {
-      const int row = 2 * it + half;
+    const uint16_t* kr = static_cast<const uint16_t*>(a.k) + (int64_t)b * a.k_sb + (int64_t)g * a.k_sh;
+    const uint16_t* vr = static_cast<const uint16_t*>(a.v) + (int64_t)b * a.v_sb + (int64_t)g * a.v_sh;
+    const int l16 = lane & 15, hf = l16 >> 3, cc = l16 & 7;
+#pragma unroll 4
+    for (int i = 0; i < 16; ++i) {
+      const int row = 2 * i + (lane >> 4);
       const int j = __shfl_sync(0xffffffffu, jj, row);
+      const uint32_t off = hf * kHalfBytes + row * 128 + ((cc ^ (row & 7)) << 4);
       if (j >= 0) {
-        cp_async16(sk + row * kRowBytes + l16 * 16, kr + (int64_t)j * a.k_sn);
-        cp_async16(sk + (kBatch + row) * kRowBytes + l16 * 16, vr + (int64_t)j * a.v_sn);
+        cp_async16(sk + off, kr + (int64_t)j * a.k_sn + l16 * 8);
+        cp_async16(sk + 2 * kHalfBytes + off, vr + (int64_t)j * a.v_sn + l16 * 8);
+      } else {
+        sts128_zero(sk + off);
+        sts128_zero(sk + 2 * kHalfBytes + off);
       }
     }
-    const uint16_t* qr = qbase + (int64_t)b * a.q_sb + (int64_t)(g * G) * a.q_sh + l16 * 8;
+    const uint16_t* qr = qbase + (int64_t)b * a.q_sb + (int64_t)(g * G) * a.q_sh;
 #pragma unroll
-    for (int hh = half; hh < G; hh += 2)
-      cp_async16(sk + (2 * kBatch + hh) * kRowBytes + l16 * 16, qr + (int64_t)hh * a.q_sh);
+    for (int hh = lane >> 4; hh < G; hh += 2)
+      cp_async16(sk + 4 * kHalfBytes + hh * kRowBytes + l16 * 16, qr + (int64_t)hh * a.q_sh + l16 * 8);
     cp_async_commit();
     return vm;
   };
@@ -149,15 +166,21 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(AttnArgs
     if (t0 + 2 < t1) jnext = load_idx(t0 + 2);
   }
 
-  float m[G], l[G], o[G][8];
+  // mma.sync fragments: row grp = lane/4 of the 16-row tiles is query head
+  // grp of the group (rows >= G and 8..15 are zero); tig = lane%4.
+  const int grp = lane >> 2, tig = lane & 3;
+  const bool head_ok = grp < G;
+  // running softmax of head grp (the 4 lanes of a group hold the same values)
+  // and its output tile O[grp][nb*8 + 2*tig + {0,1}] for the 16 dim blocks nb
+  float m_run = -INFINITY, l_run = 0.f;
+  float oacc[16][4];
   auto reset = [&]() {
+    m_run = -INFINITY;
+    l_run = 0.f;
 #pragma unroll
-    for (int hh = 0; hh < G; ++hh) {
-      m[hh] = -INFINITY;
-      l[hh] = 0.f;
+    for (int nb = 0; nb < 16; ++nb)
 #pragma unroll
-      for (int e = 0; e < 8; ++e) o[hh][e] = 0.f;
-    }
+      for (int e = 0; e < 4; ++e) oacc[nb][e] = 0.f;
   };
   reset();
   int cb = -1, cg = -1;   // the (b, g) being accumulated
@@ -165,34 +188,31 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(AttnArgs
   // write the current (b, g): the output itself when this segment holds all
   // of its batches, else a partial for the combine kernel
   auto flush = [&]() {
-    const int nb = s_nbat[cb];
-    const int first = s_bstart[cb] + cg * nb;   // first batch of (cb, cg) in the list
+    const int nb_ = s_nbat[cb];
+    const int first = s_bstart[cb] + cg * nb_;   // first batch of (cb, cg) in the list
     const int per = (total + gridDim.x * kAW - 1) / (gridDim.x * kAW);
-    const bool whole = first / per == (first + nb - 1) / per;   // one segment holds it all
+    const bool whole = first / per == (first + nb_ - 1) / per;   // one segment holds it all
     const int seg = (blockIdx.x * kAW + warp) - first / per;
+    if (!head_ok) return;
+    const int h = cg * G + grp;
+    if (whole) {
+      float* op = a.out + ((int64_t)cb * a.H + h) * kHeadDim + 2 * tig;
+      const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
 #pragma unroll
-    for (int hh = 0; hh < G; ++hh) {
-      float oo[8];
+      for (int nb = 0; nb < 16; ++nb) {
+        op[nb * 8] = oacc[nb][0] * inv;
+        op[nb * 8 + 1] = oacc[nb][1] * inv;
+      }
+    } else {
+      float* pp = a.part + (((int64_t)cb * a.H + h) * a.splits + seg) * (2 + kHeadDim);
+      if (tig == 0) {
+        pp[0] = m_run;
+        pp[1] = l_run;
+      }
 #pragma unroll
-      for (int e = 0; e < 8; ++e) oo[e] = o[hh][e] + __shfl_xor_sync(0xffffffffu, o[hh][e], 16);
-      const int h = cg * G + hh;
-      if (whole) {
-        if (half == 0) {
-          float* op = a.out + ((int64_t)cb * a.H + h) * kHeadDim + l16 * 8;
-          const float inv = l[hh] > 0.f ? 1.f / l[hh] : 0.f;
-#pragma unroll
-          for (int e = 0; e < 8; ++e) op[e] = oo[e] * inv;
-        }
-      } else {
-        float* pp = a.part + (((int64_t)cb * a.H + h) * a.splits + seg) * (2 + kHeadDim);
-        if (lane == 0) {
-          pp[0] = m[hh];
-          pp[1] = l[hh];
-        }
-        if (half == 0) {
-#pragma unroll
-          for (int e = 0; e < 8; ++e) pp[2 + l16 * 8 + e] = oo[e];
-        }
+      for (int nb = 0; nb < 16; ++nb) {
+        pp[2 + nb * 8 + 2 * tig] = oacc[nb][0];
+        pp[2 + nb * 8 + 2 * tig + 1] = oacc[nb][1];
       }
     }
   };
@@ -200,8 +220,8 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(AttnArgs
   for (int t = t0; t < t1; ++t) {
     const int s = (t - t0) & 1;
     const uint32_t sk = slot0 + s * Cfg::kSlotBytes;
-    const uint32_t sv = sk + kBatch * kRowBytes;
-    const uint32_t sq = sk + 2 * kBatch * kRowBytes;
+    const uint32_t sv = sk + 2 * kHalfBytes;
+    const uint32_t sq = sk + 4 * kHalfBytes;
     int b, g, bi;
     tab.decode(t, b, g, bi);
     if (b != cb || g != cg) {
@@ -211,54 +231,98 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(AttnArgs
       cg = g;
     }
     const unsigned vm = vmask[s];
-    // batch t is the older of at most two outstanding groups
     if (t + 1 < t1) cp_async_wait<1>(); else cp_async_wait<0>();
     __syncwarp();
 
-    float qf[G][8];
+    // S^T = q . K^T: A = q (16 rows = heads), B = K rows (n = 8 tokens)
+    uint32_t qa[8][2];
 #pragma unroll
-    for (int hh = 0; hh < G; ++hh) to_float8<DT>(lds128(sq + hh * kRowBytes + l16 * 16), qf[hh]);
-    float acc[G][16];
-#pragma unroll
-    for (int it = 0; it < 16; ++it) {
-      float kf[8];
-      to_float8<DT>(lds128(sk + (2 * it + half) * kRowBytes + l16 * 16), kf);
-#pragma unroll
-      for (int hh = 0; hh < G; ++hh) {
-        float sum = 0.f;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) sum = fmaf(qf[hh][e], kf[e], sum);
-        acc[hh][it] = sum;
+    for (int kb = 0; kb < 8; ++kb) {
+      if (head_ok) {
+        const uint32_t qaddr = sq + grp * kRowBytes + (kb * 16 + tig * 2) * 2;
+        qa[kb][0] = lds32(qaddr);
+        qa[kb][1] = lds32(qaddr + 16);
+      } else {
+        qa[kb][0] = 0u;
+        qa[kb][1] = 0u;
       }
     }
-    const bool valid = (vm >> tok) & 1u;
-    float p[G];
+    float sacc[4][4];
 #pragma unroll
-    for (int hh = 0; hh < G; ++hh) {
-      const float z = half_transpose_reduce(acc[hh], lane) * kInvSqrtD;
-      const float bm = warp_max(valid ? z : -INFINITY);
-      const float mn = fmaxf(m[hh], bm);
-      const float corr = m[hh] == -INFINITY ? 0.f : expf(m[hh] - mn);
-      p[hh] = valid ? expf(z - mn) : 0.f;
-      l[hh] = l[hh] * corr + warp_sum(p[hh]);
-      m[hh] = mn;
+    for (int nb = 0; nb < 4; ++nb) {
 #pragma unroll
-      for (int e = 0; e < 8; ++e) o[hh][e] *= corr;
+      for (int e = 0; e < 4; ++e) sacc[nb][e] = 0.f;
+      const int trow = nb * 8 + (lane & 7);
+#pragma unroll
+      for (int kp = 0; kp < 4; ++kp) {
+        const int c = 4 * kp + (lane >> 3);
+        uint32_t bk[4];
+        ldmatrix_x4(sk + (c >> 3) * kHalfBytes + trow * 128 + (((c & 7) ^ (trow & 7)) << 4), bk);
+        const uint32_t a0[4] = {qa[2 * kp][0], 0u, qa[2 * kp][1], 0u};
+        const uint32_t a1[4] = {qa[2 * kp + 1][0], 0u, qa[2 * kp + 1][1], 0u};
+        mma_16816<DT>(sacc[nb], a0, bk[0], bk[1]);
+        mma_16816<DT>(sacc[nb], a1, bk[2], bk[3]);
+      }
     }
+    // online softmax of head grp over the batch's tokens nb*8 + 2*tig + {0,1}
+    float z[8];
+    float tmax = -INFINITY;
 #pragma unroll
-    for (int it = 0; it < 16; ++it) {
-      const int row = 2 * it + half;
-      const int src = (row & 1) << 4 | (row >> 1);   // lane holding token `row`
-      float w[G];
+    for (int nb = 0; nb < 4; ++nb)
 #pragma unroll
-      for (int hh = 0; hh < G; ++hh) w[hh] = __shfl_sync(0xffffffffu, p[hh], src);
-      if ((vm >> row) & 1u) {   // rows that were not gathered hold stale bytes
-        float vf[8];
-        to_float8<DT>(lds128(sv + row * kRowBytes + l16 * 16), vf);
+      for (int e = 0; e < 2; ++e) {
+        const int tkn = nb * 8 + 2 * tig + e;
+        const float v = ((vm >> tkn) & 1u) ? sacc[nb][e] * kInvSqrtD : -INFINITY;
+        z[nb * 2 + e] = v;
+        tmax = fmaxf(tmax, v);
+      }
+    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
+    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
+    const float mn = fmaxf(m_run, tmax);
+    const float corr = (m_run == -INFINITY) ? 0.f : expf(m_run - mn);
+    float p[8], psum = 0.f;
 #pragma unroll
-        for (int hh = 0; hh < G; ++hh)
+    for (int u = 0; u < 8; ++u) {
+      p[u] = (mn == -INFINITY || z[u] == -INFINITY) ? 0.f : expf(z[u] - mn);
+      psum += p[u];
+    }
+    psum += __shfl_xor_sync(0xffffffffu, psum, 1);
+    psum += __shfl_xor_sync(0xffffffffu, psum, 2);
+    l_run = l_run * corr + psum;
+    m_run = mn;
 #pragma unroll
-          for (int e = 0; e < 8; ++e) o[hh][e] = fmaf(w[hh], vf[e], o[hh][e]);
+    for (int nb = 0; nb < 16; ++nb) {
+      oacc[nb][0] *= corr;
+      oacc[nb][1] *= corr;
+    }
+    // O += P . V: A = P (heads x 16 tokens per k block), split into a 16-bit
+    // high part and the 16-bit residual so the weights keep ~22 bits; B = V
+    // rows read transposed (k = token, n = dim)
+    uint32_t pa[2][2][2];   // [k block][hi/lo][token pair 0-7 | 8-15]
+#pragma unroll
+    for (int kt = 0; kt < 2; ++kt)
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf) {
+        const float x = p[(2 * kt + hf) * 2], y = p[(2 * kt + hf) * 2 + 1];
+        const uint32_t hi = pack2<DT>(x, y);
+        const float2 hv = unpack2<DT>(hi);
+        pa[kt][0][hf] = hi;
+        pa[kt][1][hf] = pack2<DT>(x - hv.x, y - hv.y);
+      }
+#pragma unroll
+    for (int kt = 0; kt < 2; ++kt) {
+      const int trow = kt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+      const uint32_t ahi[4] = {pa[kt][0][0], 0u, pa[kt][0][1], 0u};
+      const uint32_t alo[4] = {pa[kt][1][0], 0u, pa[kt][1][1], 0u};
+#pragma unroll
+      for (int np = 0; np < 8; ++np) {
+        const int c = 2 * np + (lane >> 4);
+        uint32_t bv[4];
+        ldmatrix_x4_trans(sv + (c >> 3) * kHalfBytes + trow * 128 + (((c & 7) ^ (trow & 7)) << 4), bv);
+        mma_16816<DT>(oacc[2 * np], ahi, bv[0], bv[1]);
+        mma_16816<DT>(oacc[2 * np], alo, bv[0], bv[1]);
+        mma_16816<DT>(oacc[2 * np + 1], ahi, bv[2], bv[3]);
+        mma_16816<DT>(oacc[2 * np + 1], alo, bv[2], bv[3]);
       }
     }
     // the slot is free: refill it with batch t + 2, prefetch the indices of t + 3

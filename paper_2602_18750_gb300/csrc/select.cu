@@ -6,18 +6,22 @@
 // cluster of C CTAs, each holding a contiguous chunk.  The exact k-th largest
 // key is found by an MSD radix select with digits of 11, 11 and 10 bits.  In
 // each pass every CTA histograms the keys that match the digits fixed so
-// far; CTA r merges bins [r*W, (r+1)*W) of all CTAs' histograms through
-// distributed shared memory and publishes its bin total; every CTA then finds
-// the crossing bin itself by reading the owner's merged bins.  A pass ends
-// the search early when the crossing bin is taken whole.  This is the GPU
-// form of the paper's merge of chunked <position, score> blocks (Sec. 4.2):
-// the chunks stay on chip and only bin counts cross between CTAs.
+// far; with a cluster, CTA r merges bins [r*W, (r+1)*W) of all CTAs'
+// histograms through distributed shared memory and publishes its bin total.
+// The crossing bin is then found in two levels -- every warp sums its slice
+// of the bins, one warp scans the 32 slice sums and then the bins of the
+// crossing slice -- so a pass costs three block barriers.  A pass ends the
+// search early when the crossing bin is taken whole.  This is the GPU form of
+// the paper's merge of chunked <position, score> blocks (Sec. 4.2): the
+// chunks stay on chip and only bin counts cross between CTAs.
 //
 // Ties at the boundary go to the lowest token index: with tau the k-th key
 // and r_eq the number of keys equal to tau that must be taken, a token is
 // selected iff key > tau, or key == tau and fewer than r_eq keys equal to tau
-// precede it.  Output positions come from prefix counts over (CTA, thread,
-// element) in index order, so idx is ascending without a sort.
+// precede it.  Each warp owns a contiguous slice of the keys; ballots give
+// the positions inside a warp, the warp totals the positions across warps
+// (and a cluster exchange across CTAs), so idx comes out in ascending order
+// without a sort.
 #include <cooperative_groups.h>
 
 #include "hill_internal.h"
@@ -27,40 +31,11 @@ namespace cg = cooperative_groups;
 namespace hill {
 namespace {
 
-constexpr int kSelThreads = 512;
+constexpr int kSelThreads = 1024;
 constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kBins = 2048;
 constexpr int kMaxCluster = 8;
 constexpr int kChunkMax = 16384;   // keys per CTA before the cluster grows
-
-// Exclusive prefix sum over the block (thread order); *total gets the sum.
-// wsum needs kSelWarps + 1 entries.
-__device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* wsum, uint32_t* total) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint32_t x = v;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
-    if (lane >= o) x += y;
-  }
-  __syncthreads();  // wsum may still be read by a previous scan
-  if (lane == 31) wsum[warp] = x;
-  __syncthreads();
-  if (warp == 0) {
-    const uint32_t t = lane < kSelWarps ? wsum[lane] : 0u;
-    uint32_t u = t;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t y = __shfl_up_sync(0xffffffffu, u, o);
-      if (lane >= o) u += y;
-    }
-    if (lane < kSelWarps) wsum[lane] = u - t;
-    if (lane == 31) wsum[kSelWarps] = u;
-  }
-  __syncthreads();
-  *total = wsum[kSelWarps];
-  return wsum[warp] + x - v;
-}
 
 template <bool CL>
 __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) {
@@ -78,17 +53,27 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
   };
   const int b = blockIdx.y;
   const int tid = threadIdx.x;
+  const int warp = tid >> 5, lane = tid & 31;
   pdl_wait();
   pdl_launch_dependents();
 
   extern __shared__ uint32_t sm[];
-  uint32_t* keys = sm;                   // [chunk]
-  uint32_t* hist = keys + a.chunk;       // [kBins]
-  uint32_t* merged = hist + kBins;       // [kBins] (only [0, nb / C) used)
-  __shared__ uint32_t wsum[kSelWarps + 1];
+  uint32_t* keys = sm;                       // [chunk]
+  uint32_t* histbuf = keys + a.chunk;        // [2][kBins], alternate passes
+  uint32_t* merged = histbuf + 2 * kBins;    // [kBins] (cluster: this CTA's merged range)
+  __shared__ uint32_t wtot[kSelWarps];
   __shared__ uint32_t tot[kMaxCluster];
-  __shared__ uint32_t cgt[kMaxCluster], ceq[kMaxCluster];
+  __shared__ uint32_t cnt[kMaxCluster];
   __shared__ uint32_t bc[3];
+
+  // Load this CTA's chunk of keys before the lengths are known: every row
+  // below the capacity is valid memory, and rows at or beyond the length are
+  // never counted.
+  const int j_lo = r * a.chunk;
+  const int ncap = max(0, min(a.chunk, a.cap - j_lo));
+  const float* kp = a.key + (int64_t)b * a.cap + j_lo;
+  for (int i = tid; i < ncap; i += kSelThreads) keys[i] = ordered_key(kp[i]);
+  for (int i = tid; i < kBins; i += kSelThreads) histbuf[i] = 0;
 
   int len = a.lens[b];
   len = len < 0 ? 0 : (len > a.cap ? a.cap : len);
@@ -99,9 +84,7 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
     kk = a.max_k;
   }
   int32_t* out = a.idx + (int64_t)b * a.max_k;
-  const int j_lo = r * a.chunk;
-  const int j_hi = min(j_lo + a.chunk, len);
-  const int n = max(0, j_hi - j_lo);
+  const int n = max(0, min(j_lo + a.chunk, len) - j_lo);
 
   // padding and count (every path)
   for (int p = kk + r * kSelThreads + tid; p < a.max_k; p += C * kSelThreads) out[p] = -1;
@@ -111,9 +94,7 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
     for (int i = tid; i < n; i += kSelThreads) out[j_lo + i] = j_lo + i;
     return;
   }
-
-  const float* kp = a.key + (int64_t)b * a.cap + j_lo;
-  for (int i = tid; i < n; i += kSelThreads) keys[i] = ordered_key(kp[i]);
+  __syncthreads();
 
   uint32_t prefix = 0, pmask = 0;
   uint32_t remaining = (uint32_t)kk;
@@ -123,12 +104,14 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
     const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
     const int nb = pass == 2 ? 1024 : 2048;
     const uint32_t dmask = (uint32_t)nb - 1u;
-    for (int i = tid; i < nb; i += kSelThreads) hist[i] = 0;
-    __syncthreads();
+    uint32_t* hist = histbuf + (pass & 1) * kBins;
+    uint32_t* next = histbuf + ((pass & 1) ^ 1) * kBins;
     for (int i = tid; i < n; i += kSelThreads) {
       const uint32_t kv = keys[i];
       if ((kv & pmask) == prefix) atomicAdd(&hist[(kv >> shift) & dmask], 1u);
     }
+    // the other buffer was last read before the previous pass ended
+    for (int i = tid; i < kBins; i += kSelThreads) next[i] = 0;
     csync();  // (A) every local histogram is complete
 
     int W = nb;
@@ -138,17 +121,19 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
     if (CL) {
       W = nb / C;
       const int base = r * W;
-      uint32_t part = 0;
       for (int i = tid; i < W; i += kSelThreads) {
         uint32_t s = 0;
         for (int c = 0; c < C; ++c) s += remote(hist, c)[base + i];
         merged[i] = s;
-        part += s;
       }
-      uint32_t mine;
-      (void)block_excl_scan(part, wsum, &mine);
-      if (tid == 0)
-        for (int c = 0; c < C; ++c) remote(tot, c)[r] = mine;
+      __syncthreads();
+      if (warp == 0) {
+        uint32_t s = 0;
+        for (int i = lane; i < W; i += 32) s += merged[i];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (lane < C) remote(tot, lane)[r] = s;
+      }
       csync();  // (B) merged bins and totals published; remote histogram reads done
       // which CTA's bin range holds the remaining-th largest matching key?
       for (int c = C - 1; c >= 0; --c) {
@@ -160,25 +145,49 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
       }
       om = remote(merged, owner);
     }
-    // positions p = 0.. run over the owner's bins from the top down
-    const int per = (W + kSelThreads - 1) / kSelThreads;
-    const int p0 = tid * per;
-    const int p1 = min(p0 + per, W);
-    uint32_t s = 0;
-    for (int p = p0; p < p1; ++p) s += om[W - 1 - p];
-    uint32_t tall;
-    const uint32_t ex = block_excl_scan(s, wsum, &tall);
-    if (above + ex < remaining && remaining <= above + ex + s) {
-      uint32_t cum = above + ex;
-      for (int p = p0; p < p1; ++p) {
-        const uint32_t c = om[W - 1 - p];
-        if (cum + c >= remaining) {
-          bc[0] = (uint32_t)(owner * W + W - 1 - p);
-          bc[1] = remaining - cum;
-          bc[2] = c;
+    // Two-level search over positions p = 0..W-1 (the owner's bins from the
+    // top down): warp w sums positions [w*S, (w+1)*S), then warp 0 scans the
+    // 32 sums and the positions of the crossing slice.
+    const int S = W / kSelWarps;   // a power of two, at least 4
+    {
+      uint32_t s = 0;
+      for (int p = warp * S + lane; p < (warp + 1) * S; p += 32) s += om[W - 1 - p];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+      if (lane == 0) wtot[warp] = s;
+    }
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t t = wtot[lane];
+      uint32_t inc = t;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+      }
+      const uint32_t need = remaining - above;   // >= 1
+      const unsigned hit = __ballot_sync(0xffffffffu, inc >= need);
+      const int ws = hit ? __ffs(hit) - 1 : 31;    // slice holding the crossing
+      uint32_t cum = __shfl_sync(0xffffffffu, inc - t, ws);
+      for (int p0 = ws * S; p0 < (ws + 1) * S; p0 += 32) {
+        const int p = p0 + lane;
+        const uint32_t c = p < (ws + 1) * S ? om[W - 1 - p] : 0u;
+        uint32_t ci = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t y = __shfl_up_sync(0xffffffffu, ci, o);
+          if (lane >= o) ci += y;
+        }
+        const unsigned h = __ballot_sync(0xffffffffu, cum + ci >= need);
+        if (h) {
+          if (lane == __ffs(h) - 1) {
+            bc[0] = (uint32_t)(owner * W + W - 1 - p);
+            bc[1] = need - (cum + ci - c);
+            bc[2] = c;
+          }
           break;
         }
-        cum += c;
+        cum += __shfl_sync(0xffffffffu, ci, 31);
       }
     }
     __syncthreads();
@@ -194,55 +203,63 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
   // bucket and above); otherwise tau = prefix is the k-th key itself and
   // `remaining` of the keys equal to tau are taken, lowest index first.
   const uint32_t tau = prefix;
+  auto is_gt = [&](uint32_t kv) { return take_bucket ? kv >= tau : kv > tau; };
+  auto is_eq = [&](uint32_t kv) { return !take_bucket && kv == tau; };
 
   // ---------------------------------------------------------------- compaction
-  const int per = (n + kSelThreads - 1) / kSelThreads;
-  const int i0 = tid * per, i1 = min(i0 + per, n);
+  // warp w owns keys [w*per, (w+1)*per), read 32 at a time; counts packed as
+  // (above tau) << 16 | (equal to tau) -- a chunk holds fewer than 2^16 keys
+  const int per = ((n + kSelWarps - 1) / kSelWarps + 31) & ~31;
+  const int w0 = min(n, warp * per), w1 = min(n, w0 + per);
   uint32_t my_gt = 0, my_eq = 0;
-  for (int i = i0; i < i1; ++i) {
+  for (int i = w0 + lane; i < w1; i += 32) {
     const uint32_t kv = keys[i];
-    if (take_bucket) {
-      my_gt += kv >= tau;
-    } else {
-      my_gt += kv > tau;
-      my_eq += kv == tau;
-    }
+    my_gt += is_gt(kv);
+    my_eq += is_eq(kv);
   }
-  uint32_t tgt, teq;
-  const uint32_t gt_ex = block_excl_scan(my_gt, wsum, &tgt);
-  const uint32_t eq_ex = block_excl_scan(my_eq, wsum, &teq);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    my_gt += __shfl_xor_sync(0xffffffffu, my_gt, o);
+    my_eq += __shfl_xor_sync(0xffffffffu, my_eq, o);
+  }
+  if (lane == 0) wtot[warp] = (my_gt << 16) | my_eq;
+  __syncthreads();
+  // prefix of the warp totals of this CTA, and the CTA total
+  uint32_t wex = 0, ctot = 0;
+  for (int w = 0; w < kSelWarps; ++w) {
+    const uint32_t t = wtot[w];
+    wex += w < warp ? t : 0u;
+    ctot += t;
+  }
   if (CL) {
     if (tid == 0)
-      for (int c = 0; c < C; ++c) {
-        remote(cgt, c)[r] = tgt;
-        remote(ceq, c)[r] = teq;
-      }
+      for (int c = 0; c < C; ++c) remote(cnt, c)[r] = ctot;
     csync();
   }
   uint32_t gt_before = 0, eq_before = 0;
   for (int c = 0; c < r; ++c) {
-    gt_before += cgt[c];
-    eq_before += ceq[c];
+    gt_before += cnt[c] >> 16;
+    eq_before += cnt[c] & 0xffffu;
   }
-  uint32_t eq_rank = eq_before + eq_ex;   // ties before this thread's segment
-  uint32_t pos = gt_before + gt_ex + min(eq_rank, remaining);
-  for (int i = i0; i < i1; ++i) {
-    const uint32_t kv = keys[i];
-    bool take;
-    if (take_bucket) {
-      take = kv >= tau;
-    } else {
-      take = kv > tau;
-      if (kv == tau) {
-        take = eq_rank < remaining;
-        ++eq_rank;
-      }
-    }
+  uint32_t eq_rank = eq_before + (wex & 0xffffu);   // ties before this warp's slice
+  uint32_t pos = gt_before + (wex >> 16) + min(eq_rank, remaining);
+  const unsigned below = (1u << lane) - 1u;
+  for (int i0 = w0; i0 < w1; i0 += 32) {
+    const int i = i0 + lane;
+    const uint32_t kv = i < w1 ? keys[i] : 0u;
+    const bool g = i < w1 && is_gt(kv);
+    const bool e = i < w1 && is_eq(kv);
+    const unsigned em = __ballot_sync(0xffffffffu, e);
+    const uint32_t my_rank = eq_rank + __popc(em & below);
+    const bool take = g || (e && my_rank < remaining);
+    const unsigned tm = __ballot_sync(0xffffffffu, take);
     if (take) {
-      if (pos < (uint32_t)kk) out[pos] = j_lo + i;
+      const uint32_t p = pos + __popc(tm & below);
+      if (p < (uint32_t)kk) out[p] = j_lo + i;
       else raise_error(a.err, kErrDevArg);   // cannot happen: more picks than the budget
-      ++pos;
     }
+    pos += __popc(tm);
+    eq_rank += __popc(em);
   }
 }
 
@@ -256,7 +273,7 @@ int select_cluster_size(int cap) {
 
 size_t select_smem_bytes(int cap, int C) {
   const int chunk = (cap + C - 1) / C;
-  return (size_t)chunk * 4 + 2 * kBins * 4;
+  return (size_t)chunk * 4 + 3 * kBins * 4;
 }
 
 cudaError_t launch_select(const SelectArgs& a0, cudaStream_t st) {
