@@ -137,7 +137,8 @@ hill_status check_desc(const hill_desc* d) {
 }
 
 struct Layout {
-  size_t scores, logits, partials, attn_part, total;
+  size_t scores, logits, partials, hist0, attn_part, total;
+  bool has_hist0;
   int score_grid, attn_grid, splits;
 };
 
@@ -162,6 +163,11 @@ Layout layout_for(const hill_desc* d, int mode, int max_k, int sms) {
   if (mode == HILL_SCORE_ATTN) off += align_up(B * H * cap * sizeof(float));
   L.partials = off;
   if (mode == HILL_SCORE_ATTN) off += align_up(B * (size_t)L.score_grid * H * sizeof(float2));
+  // leading-digit histogram of the selection key, built by the ATTN
+  // normalisation when a selection follows (max_k > 0)
+  L.hist0 = off;
+  L.has_hist0 = mode == HILL_SCORE_ATTN && max_k > 0;
+  if (L.has_hist0) off += align_up(B * (size_t)select_hist_bins() * sizeof(uint32_t));
   L.attn_part = off;
   off += align_up(B * H * (size_t)L.splits * (2 + kHeadDim) * sizeof(float));
   L.total = off + kAlign;  // room to align the caller's base pointer
@@ -177,7 +183,7 @@ hill_status from_cuda(cudaError_t e) { return e == cudaSuccess ? HILL_OK : HILL_
 
 hill_status run_score(const hill_desc* d, const void* q, const void* k, const int32_t* lens, int mode,
                       float* scores, float* accum, unsigned char* base, const Layout& L,
-                      const DeviceInfo& di, cudaStream_t st) {
+                      const DeviceInfo& di, cudaStream_t st, uint32_t* hist0 = nullptr) {
   if (d->batch == 0 || d->capacity == 0) return HILL_OK;
   const int G = d->num_q_heads / d->num_kv_heads;
   ScoreArgs a{};
@@ -204,6 +210,8 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   } else {
     a.logits = reinterpret_cast<float*>(base + L.logits);
     a.partials = reinterpret_cast<float2*>(base + L.partials);
+    a.hist0 = hist0;
+    a.hist0_words = (int64_t)d->batch * select_hist_bins();
   }
   hill_status s = from_cuda(counted(launch_score(a, d->dtype, G, raw, L.score_grid, st), 1));
   if (s != HILL_OK || raw) return s;
@@ -217,11 +225,13 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   f.nslot = L.score_grid;
   f.scores = scores;
   f.accum = accum;
+  f.hist0 = hist0;
   return from_cuda(counted(launch_attn_finalize(f, st), 1));
 }
 
 hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens, const int32_t* k,
-                       int max_k, int32_t* idx, int32_t* count, const DeviceInfo& di, cudaStream_t st) {
+                       int max_k, int32_t* idx, int32_t* count, const DeviceInfo& di, cudaStream_t st,
+                       const uint32_t* hist0 = nullptr) {
   if (d->batch == 0) return HILL_OK;
   SelectArgs a{};
   a.key = key;
@@ -232,6 +242,7 @@ hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens
   a.max_k = max_k;
   a.idx = idx;
   a.count = count;
+  a.hist0 = hist0;
   a.err = di.err;
   return from_cuda(counted(launch_select(a, st), 1));
 }
@@ -361,10 +372,12 @@ hill_status hill_evict_step(const hill_desc* desc, const void* q, const void* k_
   unsigned char* base = ws_base(ws);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* s_out = scores ? scores : (accum ? nullptr : reinterpret_cast<float*>(base + L.scores));
-  s = run_score(desc, q, k_cache, lens, mode, s_out, accum, base, L, di, st);
+  // ATTN: the normalisation also counts the leading key digit for the selection
+  uint32_t* hist0 = L.has_hist0 ? reinterpret_cast<uint32_t*>(base + L.hist0) : nullptr;
+  s = run_score(desc, q, k_cache, lens, mode, s_out, accum, base, L, di, st, hist0);
   if (s != HILL_OK) return s;
   const float* key = accum ? accum : s_out;
-  s = run_select(desc, key, lens, k, max_k, idx, count, di, st);
+  s = run_select(desc, key, lens, k, max_k, idx, count, di, st, hist0);
   if (s != HILL_OK || !out) return s;
   return run_attn(desc, q, k_cache, v_cache, idx, count, max_k, out, base, L, di, st);
 }

@@ -14,6 +14,8 @@ constexpr int kHeadDim = 128;
 constexpr int kRowBytes = kHeadDim * 2;      // one K/V row of 16-bit elements
 constexpr int kLanesPerRow = kRowBytes / 16; // 16 lanes x 16 B cover one row
 constexpr float kInvSqrtD = 0.0883883476483184405501f;  // 1 / sqrt(128)
+constexpr float kLog2eInvSqrtD = 0.12751743082459868f;     // log2(e) / sqrt(128)
+constexpr float kNegHuge = -3.402823466e38f;               // -FLT_MAX: "no value yet" in running maxima
 
 // Device error word bits (reported by hill_sync_status).
 constexpr unsigned kErrTimeout = 1u;  // a bounded wait expired
@@ -145,6 +147,15 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const void* tmap, int 
       " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(dst),
       "l"(tmap), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar), "l"(policy)
       : "memory");
+}
+
+// 2^x on the special-function unit (ex2.approx.ftz.f32, relative error about
+// 2^-22; 2^-inf = +0).  Softmax weights are formed as 2^(z*log2(e) - m) with
+// the logits kept pre-scaled by log2(e), which equals e^(z - m').
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 __device__ __forceinline__ void prefetch_tmap(const void* tmap) {

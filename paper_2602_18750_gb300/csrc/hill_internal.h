@@ -22,8 +22,10 @@ struct ScoreArgs {
   float* scores;      // RAW: per-token sums, may be NULL when accum is given
   float* accum;       // RAW: running importance (+=), may be NULL
   float* logits;      // ATTN: [B][H][cap]
-  float2* partials;   // ATTN: [B][nslot][H] (max, sum exp)
+  float2* partials;   // ATTN: [B][nslot][H] (max, sum 2^(z2 - max)), base-2 logits z2 = z * log2 e
   int nslot;          // = grid size of the launch
+  uint32_t* hist0;    // optional: zero-filled here (hist0_words words) for the normalisation to count into
+  int64_t hist0_words;
   unsigned* err;
 };
 
@@ -34,6 +36,7 @@ struct FinalizeArgs {
   int B, H, cap, nslot;
   float* scores;      // may be NULL when accum is given
   float* accum;       // may be NULL
+  uint32_t* hist0;    // optional [B][2048]: counts of the leading 11-bit digit of the selection key
 };
 
 struct SelectArgs {
@@ -42,6 +45,7 @@ struct SelectArgs {
   const int32_t* k;
   int B, cap, max_k;
   int chunk;          // filled by the launcher
+  const uint32_t* hist0;   // optional [B][2048]: counts of the leading 11-bit key digit
   int32_t* idx;
   int32_t* count;
   unsigned* err;
@@ -119,6 +123,7 @@ cudaError_t launch_attn_finalize(const FinalizeArgs& a, cudaStream_t st);
 // select.cu
 int select_cluster_size(int cap);
 size_t select_smem_bytes(int cap, int C);
+int select_hist_bins();
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
 
 // attn.cu

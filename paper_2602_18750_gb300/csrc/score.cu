@@ -6,8 +6,7 @@
 // dealt to the warps (g mod kNW).  Every warp streams its own (item, g)
 // sequence through a private ring of kSW shared-memory stages: lane 0 issues
 // two tiled TMA loads (dims 0-63 and 64-127 of the tile's 32 key rows, 128-
-// byte swizzle) plus a bulk copy of the G query rows of the head group, all
-// completing on the stage's mbarrier.  The warp moves a landed tile into
+// byte swizzle) completing on the stage's mbarrier.  The warp moves a landed tile into
 // registers with ldmatrix (conflict-free thanks to the swizzle), hands the
 // slot back to the copy engine for the stage kSW ahead, and computes the
 // [32 tokens x 128] . [128 x G heads] product with 16 mma.sync m16n8k16
@@ -17,12 +16,15 @@
 //   RAW : the per-token sum over heads is reduced across the warps in shared
 //         memory at the end of each item (fixed order) and written to scores
 //         (and added to accum).
-//   ATTN: every logit z = q.K/sqrt(d) is written to a [B][H][cap] buffer; per
-//         stage the warp reduces each head's tile (max, sum exp) and merges it
-//         into a running state in shared memory; when the CTA leaves a
-//         sequence the warp writes one partial per (sequence, head, CTA).
-//         hill_attn_finalize_kernel combines the partials and forms
-//         s[b,j] = sum_h exp(z[b,h,j] - m_bh) / L_bh.
+//   ATTN: every logit, pre-scaled by log2 e, is written to a [B][H][cap]
+//         buffer; each lane keeps a running (max, sum 2^(z2 - max)) of its
+//         own tokens per head in registers, and the lanes of a head are
+//         combined once, when the CTA leaves a sequence, into one partial per
+//         (sequence, head, CTA).  hill_attn_finalize_kernel combines the
+//         partials and forms s[b,j] = sum_h exp(z[b,h,j] - m_bh) / L_bh.
+//
+// The query rows of a warp's heads are held as mma B fragments in registers
+// for the whole sequence.
 #include "hill_internal.h"
 
 namespace hill {
@@ -40,15 +42,14 @@ constexpr int kKBytes = 2 * kBoxBytes;
 
 template <int G>
 struct ScoreCfg {
-  static constexpr int kSlotBytes = ((kKBytes + G * kRowBytes + 1023) / 1024) * 1024;
-  static constexpr int kSW = G <= 4 ? 3 : 2;             // stages per warp
+  static constexpr int kSlotBytes = kKBytes;               // one K tile (a multiple of 1024)
+  static constexpr int kSW = 3;                            // stages per warp
   static constexpr int kStages = kNW * kSW;
   // shared-memory layout (offsets from a 1024-byte aligned base)
   static constexpr int kOffBar = kStages * kSlotBytes;
   static constexpr int kOffTab = kOffBar + kStages * 8;
   static constexpr int kOffRed = kOffTab + 2 * kTableInts * 4;
-  static constexpr int kOffStat = kOffRed + 2 * kNW * kT * 4;
-  static constexpr int kOffFlag = kOffStat + kNW * kMaxNg * 8 * 8;
+  static constexpr int kOffFlag = kOffRed + 2 * kNW * kT * 4;
   static constexpr int kBytes = kOffFlag + 16 + 1024;        // + alignment slack
 };
 
@@ -65,17 +66,11 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// Merge two (max, sum exp) pairs.
-__device__ __forceinline__ float2 merge_ml(float2 x, float2 y) {
-  const float m = fmaxf(x.x, y.x);
-  if (m == -INFINITY) return make_float2(-INFINITY, 0.f);
-  return make_float2(m, x.y * expf(x.x - m) + y.y * expf(y.x - m));
-}
-
-// Position of a warp in its own stage sequence: item (global tile index) and
-// r (its r-th KV head of that item, g = warp + r * kNW).
+// Position of a warp in its own stage sequence: item (global tile index), r
+// (its r-th KV head of that item, g = warp + r * kNW) and b (the item's
+// sequence, advanced incrementally).
 struct Cursor {
-  int item, r;
+  int item, r, b;
 };
 
 template <int DT, int G, bool RAW>
@@ -84,6 +79,8 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   constexpr int kSlotBytes = Cfg::kSlotBytes;
   constexpr int kSW = Cfg::kSW;
   constexpr int kStages = Cfg::kStages;
+  // accumulator columns that can hold a head of the group: 2*tig (+1 when G > 1)
+  constexpr int kCols = G >= 2 ? 2 : 1;
 
   extern __shared__ unsigned char smem_raw[];
   const uint32_t raw_addr = smem_addr(smem_raw);
@@ -92,7 +89,6 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   int* tstart = reinterpret_cast<int*>(base + Cfg::kOffTab);          // [B+1] tile prefix
   int* slen = tstart + kTableInts;                                     // [B] clamped lengths
   float* red = reinterpret_cast<float*>(base + Cfg::kOffRed);          // [2][kNW][kT]
-  float2* stat = reinterpret_cast<float2*>(base + Cfg::kOffStat);      // [kNW][kMaxNg][8]
   volatile int* abort_flag = reinterpret_cast<int*>(base + Cfg::kOffFlag);
 
   const int warp = threadIdx.x >> 5;
@@ -107,6 +103,12 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   }
   pdl_wait();
   pdl_launch_dependents();
+  if (a.hist0) {   // this CTA's share of the leading-digit histogram, zeroed for the normalisation
+    const int64_t per = (a.hist0_words + gridDim.x - 1) / gridDim.x;
+    const int64_t w0 = min((int64_t)blockIdx.x * per, a.hist0_words);
+    const int64_t w1 = min(w0 + per, a.hist0_words);
+    for (int64_t w = w0 + threadIdx.x; w < w1; w += kThreads) a.hist0[w] = 0u;
+  }
   for (int b = threadIdx.x; b < B; b += kThreads) {
     int len = a.lens[b];
     if (len < 0 || len > cap) {
@@ -127,58 +129,43 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   }
   __syncthreads();
   const int n_items = tstart[B];
-  const int ng = (Hkv - warp + kNW - 1) / kNW;   // KV heads of this warp per tile
+  if ((int)blockIdx.x >= n_items) return;
+  const int ng = (Hkv - warp + kNW - 1) / kNW;   // KV heads of this warp per tile (0 .. kMaxNg)
 
   const uint64_t pol = l2_evict_first_policy();
-  const auto* qbase = static_cast<const uint16_t*>(a.q);
   const uint32_t stage0 = base_addr + warp * kSW * kSlotBytes;
   const uint32_t bar0 = base_addr + Cfg::kOffBar + warp * kSW * 8;
+  const int b_first = find_seq(tstart, B, blockIdx.x);
 
   auto advance = [&](Cursor& c) {
     if (++c.r >= ng) {
       c.r = 0;
       c.item += gridDim.x;
+      while (c.b < B - 1 && tstart[c.b + 1] <= c.item) ++c.b;
     }
   };
-  // lane 0: load stage `no` of this warp's sequence (position c) into its slot
-  auto issue = [&](const Cursor& c, uint32_t no) {
-    const int b = find_seq(tstart, B, c.item);
-    const int j0 = (c.item - tstart[b]) * kT;
+  // lane 0: load the K tile of position c into slot s
+  auto issue = [&](const Cursor& c, uint32_t s) {
+    const int j0 = (c.item - tstart[c.b]) * kT;
     const int g = warp + c.r * kNW;
-    const uint32_t s = no % kSW;
     const uint32_t fb = bar0 + s * 8;
     const uint32_t dst = stage0 + s * kSlotBytes;
-    mbar_arrive_expect_tx(fb, (uint32_t)(kKBytes + G * kRowBytes));
-    int crd[4] = {0, 0, 0, 0};
-    crd[a.kdim_tok] = j0;
-    crd[a.kdim_head] = g;
-    crd[a.kdim_seq] = b;
-    tma_load_4d(dst, &a.kmap, 0, crd[1], crd[2], crd[3], fb, pol);
-    tma_load_4d(dst + kBoxBytes, &a.kmap, 64, crd[1], crd[2], crd[3], fb, pol);
-    const uint16_t* qsrc = qbase + (int64_t)b * a.q_sb + (int64_t)(g * G) * a.q_sh;
-    const uint32_t qdst = dst + kKBytes;
-    if (a.q_sh == kHeadDim) {
-      bulk_g2s(qdst, qsrc, G * kRowBytes, fb);
-    } else {
-#pragma unroll
-      for (int r = 0; r < G; ++r) bulk_g2s(qdst + r * kRowBytes, qsrc + (int64_t)r * a.q_sh, kRowBytes, fb);
-    }
-  };
-
-  // per-warp running (max, sum exp) of each (stage slot r, head) of the current sequence
-  float2* wstat = stat + warp * kMaxNg * 8;
-  auto reset_stat = [&]() {
-    __syncwarp();
-    wstat[lane] = make_float2(-INFINITY, 0.f);   // kMaxNg * 8 == 32 entries
-    __syncwarp();
+    mbar_arrive_expect_tx(fb, (uint32_t)kKBytes);
+    // tensor-map coordinates: dimension 0 is d, the others are ordered by stride
+    const int c1 = a.kdim_tok == 1 ? j0 : (a.kdim_head == 1 ? g : c.b);
+    const int c2 = a.kdim_tok == 2 ? j0 : (a.kdim_head == 2 ? g : c.b);
+    const int c3 = a.kdim_tok == 3 ? j0 : (a.kdim_head == 3 ? g : c.b);
+    tma_load_4d(dst, &a.kmap, 0, c1, c2, c3, fb, pol);
+    tma_load_4d(dst + kBoxBytes, &a.kmap, 64, c1, c2, c3, fb, pol);
   };
 
   // prologue: the first kSW stages of this warp
-  Cursor pc{(int)blockIdx.x, 0};
-  uint32_t issued = 0;
+  Cursor pc{(int)blockIdx.x, 0, b_first};
+  uint32_t issued = 0, is_slot = 0;
   if (ng > 0) {
     for (; issued < (uint32_t)kSW && pc.item < n_items; ++issued) {
-      if (lane == 0) issue(pc, issued);
+      if (lane == 0) issue(pc, is_slot);
+      is_slot = is_slot + 1 == (uint32_t)kSW ? 0u : is_slot + 1;
       advance(pc);
     }
   }
@@ -186,54 +173,91 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   // fragment coordinates (mma.sync m16n8k16): C row = token lane/4 (+8),
   // C columns = heads 2*(lane%4) and 2*(lane%4)+1 of the group
   const int grp = lane >> 2, tig = lane & 3;
-  const int hA = 2 * tig, hB = 2 * tig + 1;
   // ldmatrix row address pieces: matrix m = lane/8 covers rows (m&1)*8.., k half m>>1
   const int lm_row = (lane & 7) + ((lane >> 3) & 1) * 8;
   const int lm_khalf = lane >> 4;
-  uint32_t used = 0;                       // stages consumed
+  uint32_t used = 0, cs = 0, cph = 0;      // stages consumed; slot and phase of the next one
   int item_no = 0;
   bool ok = true;
   int cur_b = -1, cur_slot = 0;
-  if (!RAW) reset_stat();
 
-  auto flush = [&]() {
-    if constexpr (!RAW) {
-      __syncwarp();
-      if (lane < ng * G) {
-        const int r = lane / G, hl = lane % G;
-        const int h = (warp + r * kNW) * G + hl;
-        a.partials[((int64_t)cur_b * a.nslot + cur_slot) * H + h] = wstat[r * 8 + hl];
+  // q of this warp's heads for the current sequence, as mma B fragments:
+  // column grp is query head g*G + grp (zero for grp >= G), k = 16*kb + 2*tig (+8)
+  uint32_t bq[kMaxNg][8][2];
+  auto load_q = [&](int b) {
+    const auto* q32 = static_cast<const uint32_t*>(a.q);
+#pragma unroll
+    for (int r = 0; r < kMaxNg; ++r) {
+      const bool has = r < ng && grp < G;
+      const int64_t row = has ? ((int64_t)b * a.q_sb + (int64_t)((warp + r * kNW) * G + grp) * a.q_sh) / 2 : 0;
+#pragma unroll
+      for (int kb = 0; kb < 8; ++kb) {
+        bq[r][kb][0] = has ? __ldg(q32 + row + kb * 8 + tig) : 0u;
+        bq[r][kb][1] = has ? __ldg(q32 + row + kb * 8 + 4 + tig) : 0u;
       }
-      __syncwarp();
+    }
+  };
+  // ATTN: this lane's running (max, sum 2^(z2 - max)) over its own tokens of
+  // the current sequence, per KV head r and column c (z2 = logit * log2 e);
+  // lanes are combined only when the CTA leaves the sequence
+  float st_m[kMaxNg][kCols], st_l[kMaxNg][kCols];
+  auto reset_stat = [&]() {
+#pragma unroll
+    for (int r = 0; r < kMaxNg; ++r)
+#pragma unroll
+      for (int c = 0; c < kCols; ++c) {
+        st_m[r][c] = kNegHuge;
+        st_l[r][c] = 0.f;
+      }
+  };
+  auto flush = [&]() {
+#pragma unroll
+    for (int r = 0; r < kMaxNg; ++r) {
+      if (r >= ng) break;
+      const int g = warp + r * kNW;
+#pragma unroll
+      for (int c = 0; c < kCols; ++c) {
+        float m = st_m[r][c], l = st_l[r][c];
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {   // the 8 lanes of one column
+          const float mo = __shfl_xor_sync(0xffffffffu, m, o);
+          const float lo = __shfl_xor_sync(0xffffffffu, l, o);
+          const float mn = fmaxf(m, mo);
+          l = l * ex2(m - mn) + lo * ex2(mo - mn);
+          m = mn;
+        }
+        const int hl = 2 * tig + c;
+        if (grp == 0 && hl < G)
+          a.partials[((int64_t)cur_b * a.nslot + cur_slot) * H + g * G + hl] = make_float2(m, l);
+      }
     }
   };
 
-  for (int item = blockIdx.x; item < n_items; item += gridDim.x, ++item_no) {
-    const int b = find_seq(tstart, B, item);
+  for (int item = blockIdx.x, b = b_first; item < n_items; item += gridDim.x, ++item_no) {
+    while (b < B - 1 && tstart[b + 1] <= item) ++b;
     const int tile = item - tstart[b];
     const int j0 = tile * kT;
     const int nv = min(kT, slen[b] - j0);
     float rs[4] = {0.f, 0.f, 0.f, 0.f};   // RAW: token sums of rows grp, grp+8, 16+grp, 24+grp
 
-    if (!RAW && b != cur_b) {
-      if (cur_b >= 0) flush();
-      reset_stat();
+    if (b != cur_b) {
+      if (!RAW && cur_b >= 0) flush();
+      load_q(b);
+      if (!RAW) reset_stat();
       cur_b = b;
       cur_slot = tile;   // = item - tstart[b]: this CTA's first item in b (< gridDim.x)
     }
 
-#pragma unroll 1
-    for (int r = 0; r < ng && ok; ++r) {
+#pragma unroll
+    for (int r = 0; r < kMaxNg; ++r) {
+      if (r >= ng || !ok) break;
       const int g = warp + r * kNW;
-      const int sr = r;   // running-state slot of this KV head
-      const uint32_t s = used % kSW;
-      if (!mbar_wait(bar0 + s * 8, (used / kSW) & 1u, a.err)) {
+      if (!mbar_wait(bar0 + cs * 8, cph, a.err)) {
         ok = false;
         *abort_flag = 1;
         break;
       }
-      const uint32_t sb = stage0 + s * kSlotBytes;
-      const uint32_t qb = sb + kKBytes;
+      const uint32_t sb = stage0 + cs * kSlotBytes;
       // K tile -> A fragments (2 blocks of 16 tokens x 8 blocks of 16 dims)
       uint32_t af[2][8][4];
 #pragma unroll
@@ -246,25 +270,15 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
           ldmatrix_x4(addr, af[mb][kb]);
         }
       }
-      // q rows -> B fragments (rows n >= G of the 8 columns are zero)
-      uint32_t bf[8][2];
-#pragma unroll
-      for (int kb = 0; kb < 8; ++kb) {
-        if (grp < G) {
-          const uint32_t qa = qb + grp * kRowBytes + (kb * 16 + tig * 2) * 2;
-          bf[kb][0] = lds32(qa);
-          bf[kb][1] = lds32(qa + 16);
-        } else {
-          bf[kb][0] = 0u;
-          bf[kb][1] = 0u;
-        }
-      }
       ++used;
+      cph ^= (cs + 1 == (uint32_t)kSW) ? 1u : 0u;
+      const uint32_t freed = cs;
+      cs = cs + 1 == (uint32_t)kSW ? 0u : cs + 1;
       __syncwarp();
-      if (pc.item < n_items) {
+      if (pc.item < n_items) {   // the slot just read takes the stage kSW ahead
         if (lane == 0) {
           fence_proxy_async_smem();
-          issue(pc, issued);
+          issue(pc, freed);
         }
         ++issued;
         advance(pc);
@@ -278,67 +292,38 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
 #pragma unroll
       for (int kb = 0; kb < 8; ++kb)
 #pragma unroll
-        for (int mb = 0; mb < 2; ++mb) mma_16816<DT>(acc[mb], af[mb][kb], bf[kb][0], bf[kb][1]);
+        for (int mb = 0; mb < 2; ++mb) mma_16816<DT>(acc[mb], af[mb][kb], bq[r][kb][0], bq[r][kb][1]);
 
-      // acc[mb][0|1] = token mb*16 + grp, heads hA|hB; acc[mb][2|3] = token mb*16 + grp + 8
-      if (RAW) {
+      // acc[mb][c] = token mb*16 + grp, column 2*tig + c; acc[mb][2 + c] = token
+      // mb*16 + grp + 8.  Columns >= G are zero (their q fragments are zero).
+      if constexpr (RAW) {
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
           const int mb = u >> 1, e = (u & 1) * 2;
-          float v = (hA < G ? acc[mb][e] : 0.f) + (hB < G ? acc[mb][e + 1] : 0.f);
-          v += __shfl_xor_sync(0xffffffffu, v, 1);
-          v += __shfl_xor_sync(0xffffffffu, v, 2);
-          rs[u] += v * kInvSqrtD;
+          float v = acc[mb][e];
+          if constexpr (G >= 2) v += acc[mb][e + 1];
+          if constexpr (G >= 4) v += __shfl_xor_sync(0xffffffffu, v, 1);
+          if constexpr (G >= 8) v += __shfl_xor_sync(0xffffffffu, v, 2);
+          rs[u] += v;   // complete in the tig == 0 lanes
         }
       } else {
-        float zA[4], zB[4];
-        bool tv[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int mb = u >> 1, e = (u & 1) * 2;
-          zA[u] = acc[mb][e] * kInvSqrtD;
-          zB[u] = acc[mb][e + 1] * kInvSqrtD;
-          tv[u] = (mb * 16 + grp + (u & 1) * 8) < nv;
-        }
         float* lg = a.logits + ((int64_t)b * H + g * G) * cap + j0;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int t = (u >> 1) * 16 + grp + (u & 1) * 8;
-          if (tv[u]) {
-            if (hA < G) lg[(int64_t)hA * cap + t] = zA[u];
-            if (hB < G) lg[(int64_t)hB * cap + t] = zB[u];
+        for (int c = 0; c < kCols; ++c) {
+          const int hl = 2 * tig + c;
+          float z[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int mb = u >> 1, e = (u & 1) * 2 + c;
+            const int t = mb * 16 + grp + (u & 1) * 8;
+            z[u] = t < nv ? acc[mb][e] * kLog2eInvSqrtD : -INFINITY;
+            if (t < nv && hl < G) lg[(int64_t)hl * cap + t] = z[u];
           }
+          const float mn = fmaxf(st_m[r][c], fmaxf(fmaxf(z[0], z[1]), fmaxf(z[2], z[3])));
+          st_l[r][c] = st_l[r][c] * ex2(st_m[r][c] - mn) +
+                       ((ex2(z[0] - mn) + ex2(z[1] - mn)) + (ex2(z[2] - mn) + ex2(z[3] - mn)));
+          st_m[r][c] = mn;
         }
-        // tile (max, sum exp) of heads hA and hB over the 8 lanes of this column pair
-        float mA = -INFINITY, mB = -INFINITY;
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-          if (tv[u]) {
-            mA = fmaxf(mA, zA[u]);
-            mB = fmaxf(mB, zB[u]);
-          }
-#pragma unroll
-        for (int o = 4; o < 32; o <<= 1) {
-          mA = fmaxf(mA, __shfl_xor_sync(0xffffffffu, mA, o));
-          mB = fmaxf(mB, __shfl_xor_sync(0xffffffffu, mB, o));
-        }
-        float lA = 0.f, lB = 0.f;
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-          if (tv[u]) {
-            lA += expf(zA[u] - mA);
-            lB += expf(zB[u] - mB);
-          }
-#pragma unroll
-        for (int o = 4; o < 32; o <<= 1) {
-          lA += __shfl_xor_sync(0xffffffffu, lA, o);
-          lB += __shfl_xor_sync(0xffffffffu, lB, o);
-        }
-        if (lane < 4) {
-          if (hA < G) wstat[sr * 8 + hA] = merge_ml(wstat[sr * 8 + hA], make_float2(mA, lA));
-          if (hB < G) wstat[sr * 8 + hB] = merge_ml(wstat[sr * 8 + hB], make_float2(mB, lB));
-        }
-        __syncwarp();
       }
     }
     if (RAW) {
@@ -356,6 +341,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
         float sum = 0.f;
 #pragma unroll
         for (int w = 0; w < kNW; ++w) sum += rb[w * kT + lane];
+        sum *= kInvSqrtD;
         const int64_t o = (int64_t)b * cap + j0 + lane;
         if (a.scores) a.scores[o] = sum;
         if (a.accum) a.accum[o] += sum;
@@ -372,20 +358,24 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   }
 }
 
-// Combine the per-CTA (max, sum exp) partials of every head of sequence b,
-// then s[b,j] = sum_h exp(z[b,h,j] - m_h) / L_h, one token per thread.  Both
-// phases issue all their loads before using them: the partials of a head are
-// spread over 8 threads, and each thread loads the logits of 16 heads of its
-// token at once (they were just written and are mostly L2 resident).
+// Combine the per-CTA (max, sum) partials of every head of sequence b, then
+// s[b,j] = sum_h 2^(z2[b,h,j] - m_h) / L_h, one token per thread (logits and
+// partials are in the base-2 scale z2 = z * log2 e, so each term is the
+// softmax weight e^(z - m) / sum e^(z - m)).  Both phases issue all their
+// loads before using them: the partials of a head are spread over 8 threads,
+// and each thread loads the logits of 16 heads of its token at once (they
+// were just written and are mostly L2 resident).
 constexpr int kFinThreads = 256;
 constexpr int kFinChunk = kFinThreads;
 constexpr int kFinPartThreads = 8;                 // threads combining one head
 constexpr int kFinPartMax = 32;                    // partials per thread held in registers
+constexpr int kHistBins = 2048;                    // leading 11 bits of the order-preserving key
 
 __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(FinalizeArgs a) {
   extern __shared__ float fsm[];
   float* mh = fsm;            // [H]
   float* il = fsm + a.H;      // [H]
+  uint32_t* hcount = reinterpret_cast<uint32_t*>(fsm + 2 * a.H);   // [kHistBins] when a.hist0
   pdl_wait();
   pdl_launch_dependents();
   const int b = blockIdx.y;
@@ -415,10 +405,10 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
     for (int o = kFinPartThreads / 2; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
     float l = 0.f;
 #pragma unroll
-    for (int u = 0; u < kFinPartMax; ++u) l += p[u].y > 0.f ? p[u].y * expf(p[u].x - m) : 0.f;
+    for (int u = 0; u < kFinPartMax; ++u) l += p[u].y > 0.f ? p[u].y * ex2(p[u].x - m) : 0.f;
     for (int s = sub + kFinPartMax * kFinPartThreads; s < ns; s += kFinPartThreads) {
       const float2 q = pb[(int64_t)s * a.H + h];
-      l += q.y * expf(q.x - m);
+      l += q.y > 0.f ? q.y * ex2(q.x - m) : 0.f;
     }
 #pragma unroll
     for (int o = kFinPartThreads / 2; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
@@ -427,23 +417,39 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
       il[h] = 1.f / l;
     }
   }
+  if (a.hist0)
+    for (int i = threadIdx.x; i < kHistBins; i += kFinThreads) hcount[i] = 0u;
   __syncthreads();
   const int j = jb + threadIdx.x;
-  if (j >= len) return;
-  const float* zp = a.logits + (int64_t)b * a.H * a.cap + j;
-  float s = 0.f;
-  int h = 0;
-  for (; h + 16 <= a.H; h += 16) {
-    float z[16];
+  if (j < len) {
+    const float* zp = a.logits + (int64_t)b * a.H * a.cap + j;
+    float s = 0.f;
+    int h = 0;
+    for (; h + 16 <= a.H; h += 16) {
+      float z[16];
 #pragma unroll
-    for (int u = 0; u < 16; ++u) z[u] = zp[(int64_t)(h + u) * a.cap];
+      for (int u = 0; u < 16; ++u) z[u] = zp[(int64_t)(h + u) * a.cap];
 #pragma unroll
-    for (int u = 0; u < 16; ++u) s += expf(z[u] - mh[h + u]) * il[h + u];
+      for (int u = 0; u < 16; ++u) s += ex2(z[u] - mh[h + u]) * il[h + u];
+    }
+    for (; h < a.H; ++h) s += ex2(zp[(int64_t)h * a.cap] - mh[h]) * il[h];
+    const int64_t o = (int64_t)b * a.cap + j;
+    if (a.scores) a.scores[o] = s;
+    float key = s;
+    if (a.accum) {
+      key = a.accum[o] + s;
+      a.accum[o] = key;
+    }
+    if (a.hist0) atomicAdd(&hcount[ordered_key(key) >> 21], 1u);
   }
-  for (; h < a.H; ++h) s += expf(zp[(int64_t)h * a.cap] - mh[h]) * il[h];
-  const int64_t o = (int64_t)b * a.cap + j;
-  if (a.scores) a.scores[o] = s;
-  if (a.accum) a.accum[o] += s;
+  if (a.hist0) {
+    __syncthreads();
+    uint32_t* hg = a.hist0 + (int64_t)b * kHistBins;
+    for (int i = threadIdx.x; i < kHistBins; i += kFinThreads) {
+      const uint32_t v = hcount[i];
+      if (v) atomicAdd(hg + i, v);
+    }
+  }
 }
 
 template <int DT, int G, bool RAW>
@@ -498,7 +504,8 @@ cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, int gri
 
 cudaError_t launch_attn_finalize(const FinalizeArgs& a, cudaStream_t st) {
   dim3 grid((a.cap + kFinChunk - 1) / kFinChunk, a.B);
-  return launch_pdl(hill_attn_finalize_kernel, grid, dim3(kFinThreads), 2 * a.H * sizeof(float), st, 0, a);
+  const size_t smem = 2 * a.H * sizeof(float) + (a.hist0 ? kHistBins * sizeof(uint32_t) : 0);
+  return launch_pdl(hill_attn_finalize_kernel, grid, dim3(kFinThreads), smem, st, 0, a);
 }
 
 }  // namespace hill

@@ -6,22 +6,24 @@
 // cluster of C CTAs, each holding a contiguous chunk.  The exact k-th largest
 // key is found by an MSD radix select with digits of 11, 11 and 10 bits.  In
 // each pass every CTA histograms the keys that match the digits fixed so
-// far; with a cluster, CTA r merges bins [r*W, (r+1)*W) of all CTAs'
-// histograms through distributed shared memory and publishes its bin total.
-// The crossing bin is then found in two levels -- every warp sums its slice
-// of the bins, one warp scans the 32 slice sums and then the bins of the
-// crossing slice -- so a pass costs three block barriers.  A pass ends the
-// search early when the crossing bin is taken whole.  This is the GPU form of
-// the paper's merge of chunked <position, score> blocks (Sec. 4.2): the
-// chunks stay on chip and only bin counts cross between CTAs.
+// far; after one cluster barrier every CTA adds up all C histograms through
+// distributed shared memory and searches the merged bins itself, so all CTAs
+// reach the same digit without further exchange.  The crossing bin is found
+// in two levels -- every warp sums its slice of the bins, one warp scans the
+// 32 slice sums and then the bins of the crossing slice.  A pass ends the
+// search early when the crossing bin is taken whole.  The first pass can
+// start from a histogram of the leading digit that the score normalisation
+// already accumulated (SelectArgs::hist0).  This is the GPU form of the
+// paper's merge of chunked <position, score> blocks (Sec. 4.2): the chunks
+// stay on chip and only bin counts cross between CTAs.
 //
 // Ties at the boundary go to the lowest token index: with tau the k-th key
 // and r_eq the number of keys equal to tau that must be taken, a token is
 // selected iff key > tau, or key == tau and fewer than r_eq keys equal to tau
-// precede it.  Each warp owns a contiguous slice of the keys; ballots give
-// the positions inside a warp, the warp totals the positions across warps
-// (and a cluster exchange across CTAs), so idx comes out in ascending order
-// without a sort.
+// precede it.  Every thread owns a contiguous run of keys; a block scan of
+// the per-thread counts (and a cluster exchange of the CTA totals) gives each
+// run its output position, so idx comes out in ascending order without a
+// sort.
 #include <cooperative_groups.h>
 
 #include "hill_internal.h"
@@ -36,6 +38,7 @@ constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kBins = 2048;
 constexpr int kMaxCluster = 8;
 constexpr int kChunkMax = 16384;   // keys per CTA before the cluster grows
+constexpr int kHistBufs = 3;       // one per pass: no buffer is rewritten while a peer may read it
 
 template <bool CL>
 __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) {
@@ -59,10 +62,9 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
 
   extern __shared__ uint32_t sm[];
   uint32_t* keys = sm;                       // [chunk]
-  uint32_t* histbuf = keys + a.chunk;        // [2][kBins], alternate passes
-  uint32_t* merged = histbuf + 2 * kBins;    // [kBins] (cluster: this CTA's merged range)
+  uint32_t* histbuf = keys + a.chunk;        // [kHistBufs][kBins], pass p uses buffer p
+  uint32_t* merged = histbuf + kHistBufs * kBins;   // [kBins]: the cluster's sum for this pass
   __shared__ uint32_t wtot[kSelWarps];
-  __shared__ uint32_t tot[kMaxCluster];
   __shared__ uint32_t cnt[kMaxCluster];
   __shared__ uint32_t bc[3];
 
@@ -72,8 +74,9 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
   const int j_lo = r * a.chunk;
   const int ncap = max(0, min(a.chunk, a.cap - j_lo));
   const float* kp = a.key + (int64_t)b * a.cap + j_lo;
+#pragma unroll 8
   for (int i = tid; i < ncap; i += kSelThreads) keys[i] = ordered_key(kp[i]);
-  for (int i = tid; i < kBins; i += kSelThreads) histbuf[i] = 0;
+  for (int i = tid; i < kHistBufs * kBins; i += kSelThreads) histbuf[i] = 0;
 
   int len = a.lens[b];
   len = len < 0 ? 0 : (len > a.cap ? a.cap : len);
@@ -104,57 +107,39 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
     const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
     const int nb = pass == 2 ? 1024 : 2048;
     const uint32_t dmask = (uint32_t)nb - 1u;
-    uint32_t* hist = histbuf + (pass & 1) * kBins;
-    uint32_t* next = histbuf + ((pass & 1) ^ 1) * kBins;
-    for (int i = tid; i < n; i += kSelThreads) {
-      const uint32_t kv = keys[i];
-      if ((kv & pmask) == prefix) atomicAdd(&hist[(kv >> shift) & dmask], 1u);
-    }
-    // the other buffer was last read before the previous pass ended
-    for (int i = tid; i < kBins; i += kSelThreads) next[i] = 0;
-    csync();  // (A) every local histogram is complete
-
-    int W = nb;
-    uint32_t above = 0;
-    int owner = 0;
-    const uint32_t* om = hist;
-    if (CL) {
-      W = nb / C;
-      const int base = r * W;
-      for (int i = tid; i < W; i += kSelThreads) {
-        uint32_t s = 0;
-        for (int c = 0; c < C; ++c) s += remote(hist, c)[base + i];
-        merged[i] = s;
+    uint32_t* hist = histbuf + pass * kBins;
+    const uint32_t* om = merged;
+    if (pass == 0 && a.hist0) {
+      // leading-digit counts over the whole sequence, accumulated upstream
+      const uint32_t* h0 = a.hist0 + (int64_t)b * kBins;
+      for (int i = tid; i < kBins; i += kSelThreads) merged[i] = h0[i];
+    } else {
+      for (int i = tid; i < n; i += kSelThreads) {
+        const uint32_t kv = keys[i];
+        if ((kv & pmask) == prefix) atomicAdd(&hist[(kv >> shift) & dmask], 1u);
       }
-      __syncthreads();
-      if (warp == 0) {
-        uint32_t s = 0;
-        for (int i = lane; i < W; i += 32) s += merged[i];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-        if (lane < C) remote(tot, lane)[r] = s;
-      }
-      csync();  // (B) merged bins and totals published; remote histogram reads done
-      // which CTA's bin range holds the remaining-th largest matching key?
-      for (int c = C - 1; c >= 0; --c) {
-        if (above + tot[c] >= remaining) {
-          owner = c;
-          break;
+      csync();  // every CTA's histogram of this pass is complete
+      if (CL) {
+        for (int i = tid; i < nb; i += kSelThreads) {
+          uint32_t v = 0;
+          for (int c = 0; c < C; ++c) v += remote(hist, c)[i];
+          merged[i] = v;
         }
-        above += tot[c];
+      } else {
+        om = hist;
       }
-      om = remote(merged, owner);
     }
-    // Two-level search over positions p = 0..W-1 (the owner's bins from the
-    // top down): warp w sums positions [w*S, (w+1)*S), then warp 0 scans the
-    // 32 sums and the positions of the crossing slice.
-    const int S = W / kSelWarps;   // a power of two, at least 4
+    __syncthreads();
+    // Two-level search over positions p = 0..nb-1 (bins from the top down):
+    // warp w sums positions [w*S, (w+1)*S), then warp 0 scans the 32 sums
+    // and the positions of the crossing slice.
+    const int S = nb / kSelWarps;   // 64 or 32
     {
-      uint32_t s = 0;
-      for (int p = warp * S + lane; p < (warp + 1) * S; p += 32) s += om[W - 1 - p];
+      uint32_t v = 0;
+      for (int p = warp * S + lane; p < (warp + 1) * S; p += 32) v += om[nb - 1 - p];
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-      if (lane == 0) wtot[warp] = s;
+      for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+      if (lane == 0) wtot[warp] = v;
     }
     __syncthreads();
     if (warp == 0) {
@@ -165,13 +150,13 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
         const uint32_t y = __shfl_up_sync(0xffffffffu, inc, o);
         if (lane >= o) inc += y;
       }
-      const uint32_t need = remaining - above;   // >= 1
+      const uint32_t need = remaining;   // >= 1
       const unsigned hit = __ballot_sync(0xffffffffu, inc >= need);
       const int ws = hit ? __ffs(hit) - 1 : 31;    // slice holding the crossing
       uint32_t cum = __shfl_sync(0xffffffffu, inc - t, ws);
       for (int p0 = ws * S; p0 < (ws + 1) * S; p0 += 32) {
         const int p = p0 + lane;
-        const uint32_t c = p < (ws + 1) * S ? om[W - 1 - p] : 0u;
+        const uint32_t c = om[nb - 1 - p];
         uint32_t ci = c;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -181,7 +166,7 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
         const unsigned h = __ballot_sync(0xffffffffu, cum + ci >= need);
         if (h) {
           if (lane == __ffs(h) - 1) {
-            bc[0] = (uint32_t)(owner * W + W - 1 - p);
+            bc[0] = (uint32_t)(nb - 1 - p);
             bc[1] = need - (cum + ci - c);
             bc[2] = c;
           }
@@ -207,59 +192,61 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
   auto is_eq = [&](uint32_t kv) { return !take_bucket && kv == tau; };
 
   // ---------------------------------------------------------------- compaction
-  // warp w owns keys [w*per, (w+1)*per), read 32 at a time; counts packed as
-  // (above tau) << 16 | (equal to tau) -- a chunk holds fewer than 2^16 keys
-  const int per = ((n + kSelWarps - 1) / kSelWarps + 31) & ~31;
-  const int w0 = min(n, warp * per), w1 = min(n, w0 + per);
-  uint32_t my_gt = 0, my_eq = 0;
-  for (int i = w0 + lane; i < w1; i += 32) {
+  // thread t owns keys [t*m, t*m + m) of the chunk (m odd: conflict-free
+  // strided reads); counts are packed as (above tau) << 16 | (equal to tau),
+  // a chunk holding fewer than 2^16 keys
+  const int m = ((n + kSelThreads - 1) / kSelThreads) | 1;
+  const int i0 = min(n, tid * m), i1 = min(n, i0 + m);
+  uint32_t mine = 0;
+  for (int i = i0; i < i1; ++i) {
     const uint32_t kv = keys[i];
-    my_gt += is_gt(kv);
-    my_eq += is_eq(kv);
+    mine += is_gt(kv) ? (1u << 16) : (is_eq(kv) ? 1u : 0u);
   }
+  // exclusive block scan of the packed counts
+  uint32_t inc = mine;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    my_gt += __shfl_xor_sync(0xffffffffu, my_gt, o);
-    my_eq += __shfl_xor_sync(0xffffffffu, my_eq, o);
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += y;
   }
-  if (lane == 0) wtot[warp] = (my_gt << 16) | my_eq;
+  if (lane == 31) wtot[warp] = inc;
   __syncthreads();
-  // prefix of the warp totals of this CTA, and the CTA total
-  uint32_t wex = 0, ctot = 0;
-  for (int w = 0; w < kSelWarps; ++w) {
-    const uint32_t t = wtot[w];
-    wex += w < warp ? t : 0u;
-    ctot += t;
-  }
-  if (CL) {
-    if (tid == 0)
-      for (int c = 0; c < C; ++c) remote(cnt, c)[r] = ctot;
-    csync();
-  }
-  uint32_t gt_before = 0, eq_before = 0;
-  for (int c = 0; c < r; ++c) {
-    gt_before += cnt[c] >> 16;
-    eq_before += cnt[c] & 0xffffu;
-  }
-  uint32_t eq_rank = eq_before + (wex & 0xffffu);   // ties before this warp's slice
-  uint32_t pos = gt_before + (wex >> 16) + min(eq_rank, remaining);
-  const unsigned below = (1u << lane) - 1u;
-  for (int i0 = w0; i0 < w1; i0 += 32) {
-    const int i = i0 + lane;
-    const uint32_t kv = i < w1 ? keys[i] : 0u;
-    const bool g = i < w1 && is_gt(kv);
-    const bool e = i < w1 && is_eq(kv);
-    const unsigned em = __ballot_sync(0xffffffffu, e);
-    const uint32_t my_rank = eq_rank + __popc(em & below);
-    const bool take = g || (e && my_rank < remaining);
-    const unsigned tm = __ballot_sync(0xffffffffu, take);
-    if (take) {
-      const uint32_t p = pos + __popc(tm & below);
-      if (p < (uint32_t)kk) out[p] = j_lo + i;
-      else raise_error(a.err, kErrDevArg);   // cannot happen: more picks than the budget
+  if (warp == 0) {
+    const uint32_t t = wtot[lane];
+    uint32_t wi = t;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, wi, o);
+      if (lane >= o) wi += y;
     }
-    pos += __popc(tm);
-    eq_rank += __popc(em);
+    wtot[lane] = wi - t;                       // exclusive prefix of warp totals
+    if (lane == 31) bc[0] = wi;                // the CTA total
+  }
+  __syncthreads();
+  const uint32_t before = wtot[warp] + inc - mine;   // this thread's exclusive prefix in the CTA
+  uint32_t gt_before = 0, eq_before = 0;
+  if (CL) {
+    if (tid < C) remote(cnt, tid)[r] = bc[0];
+    csync();
+    for (int c = 0; c < r; ++c) {
+      gt_before += cnt[c] >> 16;
+      eq_before += cnt[c] & 0xffffu;
+    }
+  }
+  uint32_t eq_rank = eq_before + (before & 0xffffu);   // ties before this run
+  uint32_t pos = gt_before + (before >> 16) + min(eq_rank, remaining);
+  for (int i = i0; i < i1; ++i) {
+    const uint32_t kv = keys[i];
+    bool take = is_gt(kv);
+    if (is_eq(kv)) {
+      take = eq_rank < remaining;
+      ++eq_rank;
+    }
+    if (take) {
+      if (pos < (uint32_t)kk) out[pos] = j_lo + i;
+      else raise_error(a.err, kErrDevArg);   // cannot happen: more picks than the budget
+      ++pos;
+    }
   }
 }
 
@@ -273,8 +260,10 @@ int select_cluster_size(int cap) {
 
 size_t select_smem_bytes(int cap, int C) {
   const int chunk = (cap + C - 1) / C;
-  return (size_t)chunk * 4 + 3 * kBins * 4;
+  return (size_t)chunk * 4 + (kHistBufs + 1) * kBins * 4;
 }
+
+int select_hist_bins() { return kBins; }
 
 cudaError_t launch_select(const SelectArgs& a0, cudaStream_t st) {
   SelectArgs a = a0;
