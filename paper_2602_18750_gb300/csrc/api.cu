@@ -251,6 +251,8 @@ hill_status run_attn(const hill_desc* d, const void* q, const void* k, const voi
                      const int32_t* count, int max_k, float* out, unsigned char* base, const Layout& L,
                      const DeviceInfo& di, cudaStream_t st) {
   if (d->batch == 0) return HILL_OK;
+  // the gather forms row offsets as 32-bit stride x 32-bit index products
+  if (d->k_sn > INT32_MAX || d->v_sn > INT32_MAX) return HILL_ERR_UNSUPPORTED;
   AttnArgs a{};
   a.q = q;
   a.k = k;

@@ -5,23 +5,27 @@
 // batches: (sequence b, KV head g, batch bi of 32 consecutive entries of
 // b's index list), ordered b, g, bi.  Every warp of the grid owns one
 // contiguous segment of that list and streams it through two shared-memory
-// slots.  A batch's 32 K rows and 32 V rows (tokens idx[b][32*bi + i]) and
-// the G query rows of the head group are gathered with 16-byte asynchronous
-// copies (one cp.async group per batch, a half-warp per 256-byte row) into
-// an XOR-swizzled layout that ldmatrix reads without bank conflicts; rows of
-// absent tokens are zero-filled.  The index entries of the batch after next
-// are loaded while the current one computes and are checked only when that
-// batch is issued.  (TMA alternatives were measured slower on the same
-// layout: 256-byte bulk copies per row are bound by the copy engine's
-// request rate, and tile::gather4 loads reached about 85 % of the cp.async
-// throughput; neither depends on how scattered the rows are.)
-// Both products run on mma.sync m16n8k16 with fp32 accumulation: S^T =
-// q . K^T (the G query heads are the rows, K rows read with ldmatrix), an
-// online softmax per head across the batches of one (b, g), and O += P . V
-// with V read by transposed ldmatrix; the weights P enter the tensor cores
-// as a 16-bit high part plus its 16-bit residual.  When a warp's segment
-// holds all batches of a (b, g) it writes the output; otherwise it writes a
-// partial (max, sum, o) that hill_attn_combine_kernel merges.
+// slots.  A batch's 32 K rows and 32 V rows (tokens idx[b][32*bi + i]) are
+// gathered with 16-byte asynchronous copies (one cp.async group per batch, a
+// half-warp per 256-byte row) into an XOR-swizzled layout that ldmatrix reads
+// without bank conflicts; rows of absent tokens are zero-filled by the copies
+// themselves.  The index entries of the batch after next are loaded while the
+// current one computes and are checked only when that batch is issued.  (TMA
+// alternatives were measured slower on the same layout: 256-byte bulk copies
+// per row are bound by the copy engine's request rate, and tile::gather4 loads
+// reached about 85 % of the cp.async throughput; neither depends on how
+// scattered the rows are.)
+// Both products run on mma.sync m16n8k16 with fp32 accumulation.  S = q . K^T
+// takes the G query heads of the group as the rows of A (held in registers
+// for all batches of a (b, g)) and K rows read with ldmatrix as B.  An online
+// softmax per head, in base 2 (logits scaled by log2(e)/sqrt(d)), runs across
+// the batches of one (b, g).  The output is accumulated transposed, O^T +=
+// V^T . P^T: V rows read with transposed ldmatrix form A (16 dims x 16
+// tokens), and the weights P -- already laid out as a B fragment by the S
+// accumulators -- enter as a 16-bit high part plus its 16-bit residual, so
+// every instruction covers 8 heads x 16 dims.  When a warp's segment holds
+// all batches of a (b, g) it writes the output; otherwise it writes a partial
+// (max, sum, o) that hill_attn_combine_kernel merges.
 #include "hill_internal.h"
 
 namespace hill {
@@ -34,30 +38,15 @@ constexpr int kMaxBatchAttn = 512;                   // sequences in the per-CTA
 
 constexpr int kHalfBytes = kBatch * 128;             // 32 rows x 64 dims, swizzled
 
-template <int G>
 struct AttnCfg {
-  // K dims 0-63 | K dims 64-127 | V dims 0-63 | V dims 64-127 | q rows
-  static constexpr int kSlotBytes = ((4 * kHalfBytes + G * kRowBytes + 1023) / 1024) * 1024;
-  static constexpr int kSmem = kAW * 2 * kSlotBytes + 1024;   // + alignment slack
+  // K dims 0-63 | K dims 64-127 | V dims 0-63 | V dims 64-127
+  static constexpr int kSlotBytes = 4 * kHalfBytes;
+  static constexpr int kSmem = kAW * 2 * kSlotBytes + 128;   // + alignment slack
 };
 
-// Batch list bookkeeping shared by the attention and combine kernels.
-struct BatchTable {
-  const int* bstart;   // [B + 1]: first batch of sequence b
-  const int* nbat;     // [B]: batches per (b, g)
-  int B, Hkv;
-
-  __device__ __forceinline__ void decode(int t, int& b, int& g, int& bi) const {
-    int lo = 0, hi = B;
-    while (hi - lo > 1) {
-      const int mid = (lo + hi) >> 1;
-      if (bstart[mid] <= t) lo = mid; else hi = mid;
-    }
-    b = lo;
-    const int rem = t - bstart[b];
-    g = rem / nbat[b];
-    bi = rem - g * nbat[b];
-  }
+// Position of a batch in the list: sequence, KV head, batch within (b, g).
+struct Pos {
+  int b, g, bi;
 };
 
 __device__ __forceinline__ int clamp_count(const AttnArgs& a, int b) {
@@ -74,7 +63,6 @@ __device__ __forceinline__ void warp_segment(int total, int nwarps, int w, int& 
 
 template <int DT, int G>
 __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __grid_constant__ AttnArgs a) {
-  using Cfg = AttnCfg<G>;
   extern __shared__ unsigned char asmem[];
   __shared__ int s_bstart[kMaxBatchAttn + 1];
   __shared__ int s_nbat[kMaxBatchAttn];
@@ -99,154 +87,184 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
     s_bstart[a.B] = acc;
   }
   __syncthreads();
-  const BatchTable tab{s_bstart, s_nbat, a.B, a.Hkv};
   const int total = s_bstart[a.B];
+  const int nwarps = gridDim.x * kAW;
+  const int gw = blockIdx.x * kAW + warp;
   int t0, t1;
-  warp_segment(total, gridDim.x * kAW, blockIdx.x * kAW + warp, t0, t1);
+  warp_segment(total, nwarps, gw, t0, t1);
   if (t0 >= t1) return;
 
-  const uint32_t base_addr = (smem_addr(asmem) + 1023u) & ~1023u;
-  const uint32_t slot0 = base_addr + warp * 2 * Cfg::kSlotBytes;
-  const auto* qbase = static_cast<const uint16_t*>(a.q);
+  // 128-byte aligned slots: every swizzled row is one bank-aligned line
+  const uint32_t slot0 = ((smem_addr(asmem) + 127u) & ~127u) + warp * 2 * AttnCfg::kSlotBytes;
+  const auto* kbase = static_cast<const uint16_t*>(a.k);
+  const auto* vbase = static_cast<const uint16_t*>(a.v);
+  const int ksn = (int)a.k_sn, vsn = (int)a.v_sn;   // the host checks both fit in 32 bits
 
-  // raw index entry of this lane for batch t (-1 past the count).  Nothing
-  // here depends on the loaded value, so the load stays in flight until the
-  // batch is issued one iteration later, where it is checked.
-  auto load_idx = [&](int t) -> int {
-    int b, g, bi;
-    tab.decode(t, b, g, bi);
-    const int e = bi * kBatch + lane;
-    return e < s_cnt[b] ? a.idx[(int64_t)b * a.max_k + e] : -1;
+  // position of batch t0 (binary search once), then advanced one batch at a time
+  Pos first;
+  {
+    int lo = 0, hi = a.B;
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (s_bstart[mid] <= t0) lo = mid; else hi = mid;
+    }
+    const int rem = t0 - s_bstart[lo];
+    first.b = lo;
+    first.g = rem / s_nbat[lo];
+    first.bi = rem - first.g * s_nbat[lo];
+  }
+  auto advance = [&](Pos& p) {
+    if (p.b >= a.B) return;
+    if (++p.bi >= s_nbat[p.b]) {
+      p.bi = 0;
+      if (++p.g >= a.Hkv) {
+        p.g = 0;
+        do {
+          ++p.b;
+        } while (p.b < a.B && s_nbat[p.b] == 0);
+      }
+    }
   };
-  // gather batch t into slot s: row r of the batch is token jj of lane r
-  // (-1: none, zero-filled).  A half-warp copies one 256-byte row; chunk c
-  // (16 bytes) of row r goes to 128-byte line r of half c / 8 at position
-  // (c % 8) ^ (r % 8), so the ldmatrix reads below are conflict-free.
-  auto issue = [&](int t, int s, int jj) {
-    int b, g, bi;
-    tab.decode(t, b, g, bi);
-    if (bi * kBatch + lane < s_cnt[b] && (jj < 0 || jj >= a.cap)) {
+
+  // raw index entry of this lane for the batch at p (-1 past the count).
+  // Nothing here depends on the loaded value, so the load stays in flight
+  // until the batch is issued one iteration later, where it is checked.
+  auto load_idx = [&](const Pos& p) -> int {
+    const int e = p.bi * kBatch + lane;
+    return e < s_cnt[p.b] ? a.idx[(int64_t)p.b * a.max_k + e] : -1;
+  };
+  // gather the batch at p into slot s: row r of the batch is token jj of
+  // lane r (-1: none, zero-filled).  A half-warp copies one 256-byte row;
+  // chunk c (16 bytes) of row r goes to 128-byte line r of half c / 8 at
+  // position (c % 8) ^ (r % 8), so the ldmatrix reads below are conflict-free.
+  const int l16 = lane & 15, hrow = lane >> 4;
+  const uint32_t dst_lane = (uint32_t)((l16 >> 3) * kHalfBytes + hrow * 128);
+  const uint32_t swz_lane = (uint32_t)(((l16 & 7) ^ hrow) << 4);
+  auto issue = [&](const Pos& p, int s, int jj) -> unsigned {
+    if (p.bi * kBatch + lane < s_cnt[p.b] && (jj < 0 || jj >= a.cap)) {
       raise_error(a.err, kErrDevArg);   // a listed entry outside [0, cap): skipped
       jj = -1;
     }
     const unsigned vm = __ballot_sync(0xffffffffu, jj >= 0);
-    const uint32_t sk = slot0 + s * Cfg::kSlotBytes;
-    const uint16_t* kr = static_cast<const uint16_t*>(a.k) + (int64_t)b * a.k_sb + (int64_t)g * a.k_sh;
-    const uint16_t* vr = static_cast<const uint16_t*>(a.v) + (int64_t)b * a.v_sb + (int64_t)g * a.v_sh;
-    const int l16 = lane & 15, hf = l16 >> 3, cc = l16 & 7;
-#pragma unroll 4
-    for (int i = 0; i < 16; ++i) {
-      const int row = 2 * i + (lane >> 4);
-      const int j = __shfl_sync(0xffffffffu, jj, row);
-      const uint32_t off = hf * kHalfBytes + row * 128 + ((cc ^ (row & 7)) << 4);
-      if (j >= 0) {
-        cp_async16(sk + off, kr + (int64_t)j * a.k_sn + l16 * 8);
-        cp_async16(sk + 2 * kHalfBytes + off, vr + (int64_t)j * a.v_sn + l16 * 8);
-      } else {
-        sts128_zero(sk + off);
-        sts128_zero(sk + 2 * kHalfBytes + off);
-      }
-    }
-    const uint16_t* qr = qbase + (int64_t)b * a.q_sb + (int64_t)(g * G) * a.q_sh;
+    const uint32_t sk = slot0 + s * AttnCfg::kSlotBytes + dst_lane;
+    const uint16_t* kr = kbase + (int64_t)p.b * a.k_sb + (int64_t)p.g * a.k_sh + l16 * 8;
+    const uint16_t* vr = vbase + (int64_t)p.b * a.v_sb + (int64_t)p.g * a.v_sh + l16 * 8;
 #pragma unroll
-    for (int hh = lane >> 4; hh < G; hh += 2)
-      cp_async16(sk + 4 * kHalfBytes + hh * kRowBytes + l16 * 16, qr + (int64_t)hh * a.q_sh + l16 * 8);
+    for (int i = 0; i < 16; ++i) {
+      const int j = __shfl_sync(0xffffffffu, jj, 2 * i + hrow);
+      const uint32_t nbytes = j >= 0 ? 16u : 0u;
+      const int jc = j >= 0 ? j : 0;
+      // row 2i + hrow: (2i + hrow) % 8 = (2i % 8) | hrow
+      const uint32_t off = (uint32_t)(i * 256) + (swz_lane ^ (uint32_t)(((2 * i) & 7) << 4));
+      cp_async16_zfill(sk + off, kr + (int64_t)jc * ksn, nbytes);
+      cp_async16_zfill(sk + 2 * kHalfBytes + off, vr + (int64_t)jc * vsn, nbytes);
+    }
     cp_async_commit();
     return vm;
   };
 
   // prologue: batches t0 and t0 + 1, and the indices of t0 + 2
-  unsigned vmask[2] = {0u, 0u};
+  Pos pc = first, pi = first, pl = first;
+  unsigned vm0 = 0u, vm1 = 0u;
   int jnext = -1;
   {
-    int j0 = load_idx(t0);
-    int j1 = t0 + 1 < t1 ? load_idx(t0 + 1) : -1;
-    vmask[0] = issue(t0, 0, j0);
-    if (t0 + 1 < t1) vmask[1] = issue(t0 + 1, 1, j1);
-    if (t0 + 2 < t1) jnext = load_idx(t0 + 2);
+    const int j0 = load_idx(pl);
+    advance(pl);
+    const int j1 = t0 + 1 < t1 ? load_idx(pl) : -1;
+    advance(pl);
+    vm0 = issue(pi, 0, j0);
+    advance(pi);
+    if (t0 + 1 < t1) {
+      vm1 = issue(pi, 1, j1);
+      advance(pi);
+    }
+    if (t0 + 2 < t1) jnext = load_idx(pl);
+    advance(pl);
   }
 
-  // mma.sync fragments: row grp = lane/4 of the 16-row tiles is query head
-  // grp of the group (rows >= G and 8..15 are zero); tig = lane%4.
+  // mma.sync fragments: grp = lane/4, tig = lane%4.  S accumulators: row grp
+  // = query head grp of the group (rows >= G and 8..15 are zero), columns =
+  // tokens nb*8 + 2*tig + {0,1}.  O^T accumulators: rows = dims db*16 + grp
+  // (+8), columns = heads 2*tig, 2*tig + 1.
   const int grp = lane >> 2, tig = lane & 3;
   const bool head_ok = grp < G;
-  // running softmax of head grp (the 4 lanes of a group hold the same values)
-  // and its output tile O[grp][nb*8 + 2*tig + {0,1}] for the 16 dim blocks nb
-  float m_run = -INFINITY, l_run = 0.f;
-  float oacc[16][4];
-  auto reset = [&]() {
+  const int hA = 2 * tig, hB = 2 * tig + 1;   // heads of this lane's O^T columns
+  float m_run = -INFINITY, l_run = 0.f;       // softmax state of head grp (base 2)
+  float oacc[8][4];
+  uint32_t qa[8][2];                          // q rows of the group as A fragments
+  int cb = -1, cg = -1;                       // the (b, g) being accumulated
+  const int per = (total + nwarps - 1) / nwarps;
+
+  auto reset = [&](int b, int g) {
     m_run = -INFINITY;
     l_run = 0.f;
 #pragma unroll
-    for (int nb = 0; nb < 16; ++nb)
+    for (int db = 0; db < 8; ++db)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) oacc[nb][e] = 0.f;
+      for (int e = 0; e < 4; ++e) oacc[db][e] = 0.f;
+    const auto* q32 = static_cast<const uint32_t*>(a.q);
+    const int64_t row = head_ok ? ((int64_t)b * a.q_sb + (int64_t)(g * G + grp) * a.q_sh) / 2 : 0;
+#pragma unroll
+    for (int kb = 0; kb < 8; ++kb) {
+      qa[kb][0] = head_ok ? __ldg(q32 + row + kb * 8 + tig) : 0u;
+      qa[kb][1] = head_ok ? __ldg(q32 + row + kb * 8 + 4 + tig) : 0u;
+    }
   };
-  reset();
-  int cb = -1, cg = -1;   // the (b, g) being accumulated
 
   // write the current (b, g): the output itself when this segment holds all
   // of its batches, else a partial for the combine kernel
   auto flush = [&]() {
     const int nb_ = s_nbat[cb];
-    const int first = s_bstart[cb] + cg * nb_;   // first batch of (cb, cg) in the list
-    const int per = (total + gridDim.x * kAW - 1) / (gridDim.x * kAW);
-    const bool whole = first / per == (first + nb_ - 1) / per;   // one segment holds it all
-    const int seg = (blockIdx.x * kAW + warp) - first / per;
-    if (!head_ok) return;
-    const int h = cg * G + grp;
-    if (whole) {
-      float* op = a.out + ((int64_t)cb * a.H + h) * kHeadDim + 2 * tig;
-      const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+    const int firstb = s_bstart[cb] + cg * nb_;   // first batch of (cb, cg) in the list
+    const bool whole = firstb / per == (firstb + nb_ - 1) / per;   // one segment holds it all
+    const int seg = gw - firstb / per;
+    // (max, sum) of the heads in this lane's O^T columns
+    const float mA = __shfl_sync(0xffffffffu, m_run, 8 * tig), lA = __shfl_sync(0xffffffffu, l_run, 8 * tig);
+    const float mB = __shfl_sync(0xffffffffu, m_run, 8 * tig + 4), lB = __shfl_sync(0xffffffffu, l_run, 8 * tig + 4);
 #pragma unroll
-      for (int nb = 0; nb < 16; ++nb) {
-        op[nb * 8] = oacc[nb][0] * inv;
-        op[nb * 8 + 1] = oacc[nb][1] * inv;
-      }
-    } else {
-      float* pp = a.part + (((int64_t)cb * a.H + h) * a.splits + seg) * (2 + kHeadDim);
-      if (tig == 0) {
-        pp[0] = m_run;
-        pp[1] = l_run;
-      }
+    for (int c = 0; c < 2; ++c) {
+      const int hl = c ? hB : hA;
+      if (hl >= G) continue;
+      const float m = c ? mB : mA, l = c ? lB : lA;
+      const int h = cg * G + hl;
+      if (whole) {
+        float* op = a.out + ((int64_t)cb * a.H + h) * kHeadDim + grp;
+        const float inv = l > 0.f ? 1.f / l : 0.f;
 #pragma unroll
-      for (int nb = 0; nb < 16; ++nb) {
-        pp[2 + nb * 8 + 2 * tig] = oacc[nb][0];
-        pp[2 + nb * 8 + 2 * tig + 1] = oacc[nb][1];
+        for (int db = 0; db < 8; ++db) {
+          op[db * 16] = oacc[db][c] * inv;
+          op[db * 16 + 8] = oacc[db][2 + c] * inv;
+        }
+      } else {
+        float* pp = a.part + (((int64_t)cb * a.H + h) * a.splits + seg) * (2 + kHeadDim);
+        if (grp == 0) {
+          pp[0] = m;
+          pp[1] = l;
+        }
+#pragma unroll
+        for (int db = 0; db < 8; ++db) {
+          pp[2 + db * 16 + grp] = oacc[db][c];
+          pp[2 + db * 16 + 8 + grp] = oacc[db][2 + c];
+        }
       }
     }
   };
 
   for (int t = t0; t < t1; ++t) {
     const int s = (t - t0) & 1;
-    const uint32_t sk = slot0 + s * Cfg::kSlotBytes;
+    const uint32_t sk = slot0 + s * AttnCfg::kSlotBytes;
     const uint32_t sv = sk + 2 * kHalfBytes;
-    const uint32_t sq = sk + 4 * kHalfBytes;
-    int b, g, bi;
-    tab.decode(t, b, g, bi);
-    if (b != cb || g != cg) {
+    if (pc.b != cb || pc.g != cg) {
       if (cb >= 0) flush();
-      reset();
-      cb = b;
-      cg = g;
+      cb = pc.b;
+      cg = pc.g;
+      reset(cb, cg);
     }
-    const unsigned vm = vmask[s];
+    const unsigned vm = s ? vm1 : vm0;
     if (t + 1 < t1) cp_async_wait<1>(); else cp_async_wait<0>();
     __syncwarp();
 
-    // S^T = q . K^T: A = q (16 rows = heads), B = K rows (n = 8 tokens)
-    uint32_t qa[8][2];
-#pragma unroll
-    for (int kb = 0; kb < 8; ++kb) {
-      if (head_ok) {
-        const uint32_t qaddr = sq + grp * kRowBytes + (kb * 16 + tig * 2) * 2;
-        qa[kb][0] = lds32(qaddr);
-        qa[kb][1] = lds32(qaddr + 16);
-      } else {
-        qa[kb][0] = 0u;
-        qa[kb][1] = 0u;
-      }
-    }
+    // S = q . K^T: A = q (16 rows = heads), B = K rows (n = 8 tokens)
     float sacc[4][4];
 #pragma unroll
     for (int nb = 0; nb < 4; ++nb) {
@@ -272,33 +290,39 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
         const int tkn = nb * 8 + 2 * tig + e;
-        const float v = ((vm >> tkn) & 1u) ? sacc[nb][e] * kInvSqrtD : -INFINITY;
+        const float v = ((vm >> tkn) & 1u) ? sacc[nb][e] * kLog2eInvSqrtD : -INFINITY;
         z[nb * 2 + e] = v;
         tmax = fmaxf(tmax, v);
       }
     tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
     tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
-    const float mn = fmaxf(m_run, tmax);
-    const float corr = (m_run == -INFINITY) ? 0.f : expf(m_run - mn);
+    const float mn = fmaxf(m_run, tmax);      // finite: every batch holds a token
+    const float corr = ex2(m_run - mn);       // 0 on the first batch
     float p[8], psum = 0.f;
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
-      p[u] = (mn == -INFINITY || z[u] == -INFINITY) ? 0.f : expf(z[u] - mn);
+      p[u] = head_ok ? ex2(z[u] - mn) : 0.f;
       psum += p[u];
     }
     psum += __shfl_xor_sync(0xffffffffu, psum, 1);
     psum += __shfl_xor_sync(0xffffffffu, psum, 2);
     l_run = l_run * corr + psum;
     m_run = mn;
+    // rescale O^T: columns hA, hB take the factor of their head
+    const float cA = __shfl_sync(0xffffffffu, corr, 8 * tig);
+    const float cB = __shfl_sync(0xffffffffu, corr, 8 * tig + 4);
 #pragma unroll
-    for (int nb = 0; nb < 16; ++nb) {
-      oacc[nb][0] *= corr;
-      oacc[nb][1] *= corr;
+    for (int db = 0; db < 8; ++db) {
+      oacc[db][0] *= cA;
+      oacc[db][2] *= cA;
+      if constexpr (G > 1) {
+        oacc[db][1] *= cB;
+        oacc[db][3] *= cB;
+      }
     }
-    // O += P . V: A = P (heads x 16 tokens per k block), split into a 16-bit
-    // high part and the 16-bit residual so the weights keep ~22 bits; B = V
-    // rows read transposed (k = token, n = dim)
-    uint32_t pa[2][2][2];   // [k block][hi/lo][token pair 0-7 | 8-15]
+    // P as B fragments (k = token, n = head grp), split into a 16-bit high
+    // part and its 16-bit residual so the weights keep ~22 bits
+    uint32_t pb[2][2][2];   // [k block][hi/lo][tokens 0-7 | 8-15 of the block]
 #pragma unroll
     for (int kt = 0; kt < 2; ++kt)
 #pragma unroll
@@ -306,37 +330,39 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
         const float x = p[(2 * kt + hf) * 2], y = p[(2 * kt + hf) * 2 + 1];
         const uint32_t hi = pack2<DT>(x, y);
         const float2 hv = unpack2<DT>(hi);
-        pa[kt][0][hf] = hi;
-        pa[kt][1][hf] = pack2<DT>(x - hv.x, y - hv.y);
+        pb[kt][0][hf] = hi;
+        pb[kt][1][hf] = pack2<DT>(x - hv.x, y - hv.y);
       }
+    // O^T += V^T . P^T: A = V^T (16 dims x 16 tokens) by transposed ldmatrix
 #pragma unroll
     for (int kt = 0; kt < 2; ++kt) {
-      const int trow = kt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-      const uint32_t ahi[4] = {pa[kt][0][0], 0u, pa[kt][0][1], 0u};
-      const uint32_t alo[4] = {pa[kt][1][0], 0u, pa[kt][1][1], 0u};
+      const int trow = kt * 16 + (lane & 7) + ((lane >> 4) & 1) * 8;
 #pragma unroll
-      for (int np = 0; np < 8; ++np) {
-        const int c = 2 * np + (lane >> 4);
-        uint32_t bv[4];
-        ldmatrix_x4_trans(sv + (c >> 3) * kHalfBytes + trow * 128 + (((c & 7) ^ (trow & 7)) << 4), bv);
-        mma_16816<DT>(oacc[2 * np], ahi, bv[0], bv[1]);
-        mma_16816<DT>(oacc[2 * np], alo, bv[0], bv[1]);
-        mma_16816<DT>(oacc[2 * np + 1], ahi, bv[2], bv[3]);
-        mma_16816<DT>(oacc[2 * np + 1], alo, bv[2], bv[3]);
+      for (int db = 0; db < 8; ++db) {
+        const int c = 2 * db + ((lane >> 3) & 1);
+        uint32_t av[4];
+        ldmatrix_x4_trans(sv + (c >> 3) * kHalfBytes + trow * 128 + (((c & 7) ^ (trow & 7)) << 4), av);
+        mma_16816<DT>(oacc[db], av, pb[kt][0][0], pb[kt][0][1]);
+        mma_16816<DT>(oacc[db], av, pb[kt][1][0], pb[kt][1][1]);
       }
     }
     // the slot is free: refill it with batch t + 2, prefetch the indices of t + 3
     __syncwarp();
     if (t + 2 < t1) {
-      vmask[s] = issue(t + 2, s, jnext);
-      jnext = t + 3 < t1 ? load_idx(t + 3) : -1;
+      const unsigned v = issue(pi, s, jnext);
+      if (s) vm1 = v; else vm0 = v;
+      advance(pi);
+      jnext = t + 3 < t1 ? load_idx(pl) : -1;
+      advance(pl);
     }
+    advance(pc);
   }
-  if (cb >= 0) flush();
+  flush();
 }
 
 // Merge the partials of one (b, h) whose batches were split over several
-// warps: out = sum_s e^{M_s - M} O_s / sum_s e^{M_s - M} L_s.  Pairs held
+// warps: out = sum_s 2^{M_s - M} O_s / sum_s 2^{M_s - M} L_s (maxima in the
+// base-2 scale of the attention kernel).  Pairs held
 // whole by one warp were written directly; sequences with no selected token
 // get zeros.
 __global__ void __launch_bounds__(kHeadDim) hill_attn_combine_kernel(AttnArgs a, int total_warps) {
@@ -379,7 +405,7 @@ __global__ void __launch_bounds__(kHeadDim) hill_attn_combine_kernel(AttnArgs a,
   if (M != -INFINITY) {
     for (int s = 0; s < nseg; ++s) {
       const float* q = pp + s * (2 + kHeadDim);
-      const float c = q[0] == -INFINITY ? 0.f : expf(q[0] - M);
+      const float c = ex2(q[0] - M);   // partial maxima are in the base-2 scale
       L += q[1] * c;
       O += q[2 + dd] * c;
     }
@@ -391,9 +417,9 @@ template <int DT, int G>
 cudaError_t launch_attn_t(const AttnArgs& a, int grid, cudaStream_t st) {
   static int cache[64] = {0};
   auto kern = hill_sparse_attn_kernel<DT, G>;
-  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), AttnCfg<G>::kSmem, cache);
+  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), AttnCfg::kSmem, cache);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(kern, dim3(grid), dim3(kAThreads), AttnCfg<G>::kSmem, st, 0, a);
+  e = launch_pdl(kern, dim3(grid), dim3(kAThreads), AttnCfg::kSmem, st, 0, a);
   if (e != cudaSuccess) return e;
   return launch_pdl(hill_attn_combine_kernel, dim3(a.B * a.H), dim3(kHeadDim), 0, st, 0, a, grid * kAW);
 }
