@@ -31,8 +31,9 @@
 namespace hill {
 namespace {
 
-constexpr int kAW = 6;                               // warps per CTA
+constexpr int kAW = 8;                               // warps per CTA
 constexpr int kAThreads = kAW * 32;
+constexpr int kNS = 1;                               // shared-memory slots (batches in flight) per warp
 constexpr int kBatch = 32;                           // selected entries per batch
 constexpr int kMaxBatchAttn = 512;                   // sequences in the per-CTA table
 
@@ -41,7 +42,7 @@ constexpr int kHalfBytes = kBatch * 128;             // 32 rows x 64 dims, swizz
 struct AttnCfg {
   // K dims 0-63 | K dims 64-127 | V dims 0-63 | V dims 64-127
   static constexpr int kSlotBytes = 4 * kHalfBytes;
-  static constexpr int kSmem = kAW * 2 * kSlotBytes + 128;   // + alignment slack
+  static constexpr int kSmem = kAW * kNS * kSlotBytes + 128;   // + alignment slack
 };
 
 // Position of a batch in the list: sequence, KV head, batch within (b, g).
@@ -95,7 +96,8 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   if (t0 >= t1) return;
 
   // 128-byte aligned slots: every swizzled row is one bank-aligned line
-  const uint32_t slot0 = ((smem_addr(asmem) + 127u) & ~127u) + warp * 2 * AttnCfg::kSlotBytes;
+  const uint32_t slot0 = ((smem_addr(asmem) + 127u) & ~127u) + warp * kNS * AttnCfg::kSlotBytes;
+  __shared__ unsigned s_vm[kAW][kNS];   // per slot: which rows of its batch hold a token
   const auto* kbase = static_cast<const uint16_t*>(a.k);
   const auto* vbase = static_cast<const uint16_t*>(a.v);
   const int ksn = (int)a.k_sn, vsn = (int)a.v_sn;   // the host checks both fit in 32 bits
@@ -163,22 +165,25 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
     return vm;
   };
 
-  // prologue: batches t0 and t0 + 1, and the indices of t0 + 2
+  // prologue: batches t0 .. t0 + kNS - 1, and the indices of t0 + kNS
   Pos pc = first, pi = first, pl = first;
-  unsigned vm0 = 0u, vm1 = 0u;
   int jnext = -1;
   {
-    const int j0 = load_idx(pl);
-    advance(pl);
-    const int j1 = t0 + 1 < t1 ? load_idx(pl) : -1;
-    advance(pl);
-    vm0 = issue(pi, 0, j0);
-    advance(pi);
-    if (t0 + 1 < t1) {
-      vm1 = issue(pi, 1, j1);
-      advance(pi);
+    int jq[kNS];
+#pragma unroll
+    for (int u = 0; u < kNS; ++u) {
+      jq[u] = t0 + u < t1 ? load_idx(pl) : -1;
+      advance(pl);
     }
-    if (t0 + 2 < t1) jnext = load_idx(pl);
+#pragma unroll
+    for (int u = 0; u < kNS; ++u) {
+      if (t0 + u < t1) {
+        const unsigned v = issue(pi, u, jq[u]);
+        if (lane == 0) s_vm[warp][u] = v;
+        advance(pi);
+      }
+    }
+    if (t0 + kNS < t1) jnext = load_idx(pl);
     advance(pl);
   }
 
@@ -251,7 +256,7 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   };
 
   for (int t = t0; t < t1; ++t) {
-    const int s = (t - t0) & 1;
+    const int s = (t - t0) % kNS;
     const uint32_t sk = slot0 + s * AttnCfg::kSlotBytes;
     const uint32_t sv = sk + 2 * kHalfBytes;
     if (pc.b != cb || pc.g != cg) {
@@ -260,9 +265,14 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
       cg = pc.g;
       reset(cb, cg);
     }
-    const unsigned vm = s ? vm1 : vm0;
-    if (t + 1 < t1) cp_async_wait<1>(); else cp_async_wait<0>();
+    // batch t is complete once at most min(kNS - 1, t1 - 1 - t) later groups are pending
+    const int later = min(kNS - 1, t1 - 1 - t);
+    if (later >= kNS - 1) cp_async_wait<kNS - 1>();
+    else if (kNS > 2 && later == 2) cp_async_wait<(kNS > 2 ? 2 : 0)>();
+    else if (later == 1) cp_async_wait<1>();
+    else cp_async_wait<0>();
     __syncwarp();
+    const unsigned vm = s_vm[warp][s];
 
     // S = q . K^T: A = q (16 rows = heads), B = K rows (n = 8 tokens)
     float sacc[4][4];
@@ -346,13 +356,13 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
         mma_16816<DT>(oacc[db], av, pb[kt][1][0], pb[kt][1][1]);
       }
     }
-    // the slot is free: refill it with batch t + 2, prefetch the indices of t + 3
+    // the slot is free: refill it with batch t + kNS, prefetch the indices of t + kNS + 1
     __syncwarp();
-    if (t + 2 < t1) {
+    if (t + kNS < t1) {
       const unsigned v = issue(pi, s, jnext);
-      if (s) vm1 = v; else vm0 = v;
+      if (lane == 0) s_vm[warp][s] = v;
       advance(pi);
-      jnext = t + 3 < t1 ? load_idx(pl) : -1;
+      jnext = t + kNS + 1 < t1 ? load_idx(pl) : -1;
       advance(pl);
     }
     advance(pc);

@@ -370,6 +370,7 @@ constexpr int kFinChunk = kFinThreads;
 constexpr int kFinPartThreads = 8;                 // threads combining one head
 constexpr int kFinPartMax = 32;                    // partials per thread held in registers
 constexpr int kHistBins = 2048;                    // leading 11 bits of the order-preserving key
+constexpr int kFinZReg = 32;                       // logits per token held in registers
 
 __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(FinalizeArgs a) {
   extern __shared__ float fsm[];
@@ -383,6 +384,14 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   len = len < 0 ? 0 : (len > a.cap ? a.cap : len);
   const int jb = blockIdx.x * kFinChunk;
   if (jb >= len) return;
+  // this token's logits of the first kFinZReg heads, loaded before the
+  // partials are combined so that both round trips overlap
+  const int j = jb + threadIdx.x;
+  const bool valid = j < len;
+  const float* zp = a.logits + (int64_t)b * a.H * a.cap + j;
+  float zr[kFinZReg];
+#pragma unroll
+  for (int u = 0; u < kFinZReg; ++u) zr[u] = (valid && u < a.H) ? zp[(int64_t)u * a.cap] : 0.f;
   const int items = (len + kT - 1) / kT;
   const int ns = min(items, a.nslot);
   const float2* pb = a.partials + (int64_t)b * a.nslot * a.H;
@@ -420,11 +429,12 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   if (a.hist0)
     for (int i = threadIdx.x; i < kHistBins; i += kFinThreads) hcount[i] = 0u;
   __syncthreads();
-  const int j = jb + threadIdx.x;
-  if (j < len) {
-    const float* zp = a.logits + (int64_t)b * a.H * a.cap + j;
+  if (valid) {
     float s = 0.f;
-    int h = 0;
+#pragma unroll
+    for (int u = 0; u < kFinZReg; ++u)
+      if (u < a.H) s += ex2(zr[u] - mh[u]) * il[u];
+    int h = kFinZReg;
     for (; h + 16 <= a.H; h += 16) {
       float z[16];
 #pragma unroll
