@@ -14,6 +14,7 @@ arrays into it.  Each wrapper names the part of the paper it follows:
                           Sec. 4.4 (raw inner product, RAW)
 * :func:`accumulate`   -- running importance across decode steps (Sec. 4.2)
 * :func:`topk`         -- top-alpha selection (Sec. 3.1, Sec. 4.2)
+* :func:`bkp_select`   -- BKP pinning + hit-rate table (Sec. 4.2)
 * :func:`sparse_attn`  -- attention over the selected KV only (Sec. 4.1, workflow step 6)
 * :func:`evict_step`   -- the five steps in order
 
@@ -75,6 +76,7 @@ def _load():
             lib.oracle_scores.argtypes = [I, I, I, I, P, P, P]
             lib.oracle_accumulate.argtypes = [I, I, P, P, P]
             lib.oracle_topk.argtypes = [I, I, P, P, P, I, P, P]
+            lib.oracle_bkp_select.argtypes = [I, I, P, P, P, I, I, P, P, P]
             lib.oracle_sparse_attn.argtypes = [I, I, I, I, I, I, P, P, P, P, P, I, P]
             lib.oracle_evict_step.argtypes = [I, I, I, I, I, I, I, P, P, P, P, P, I,
                                               P, P, P, P, P, P]
@@ -178,6 +180,20 @@ def topk(key, lens, k, max_k):
     rc = _load().oracle_topk(B, cap, _ptr(_i32(lens)), _ptr(key), _ptr(_i32(k)), max_k,
                              _ptr(idx), _ptr(count))
     return idx, count, rc
+
+
+def bkp_select(key, lens, k, recent, max_k, hits=None):
+    """BKP selection (Sec. 4.2): pinned recent window + top-k of the older
+    tokens.  Returns (idx[B][max_k], count[B], rc, hits') with hits' a
+    uint16 copy of `hits` after the step's increments (None if hits is None)."""
+    key = np.ascontiguousarray(key, dtype=np.float64)
+    B, cap = key.shape
+    idx = np.full((B, max_k), -7, dtype=np.int32)
+    count = np.zeros(B, dtype=np.int32)
+    h = None if hits is None else np.array(hits, dtype=np.uint16, copy=True, order="C")
+    rc = _load().oracle_bkp_select(B, cap, _ptr(_i32(lens)), _ptr(key), _ptr(_i32(k)), int(recent),
+                                   max_k, _ptr(idx), _ptr(count), _ptr(h))
+    return idx, count, rc, h
 
 
 def sparse_attn(q, K, V, idx, count, dtype=None) -> np.ndarray:

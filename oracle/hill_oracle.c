@@ -221,6 +221,64 @@ int oracle_topk(int B, int cap, const int32_t* lens, const double* key,
 }
 
 /*
+ * BKP bookkeeping (Sec. 4.2, "Bidirectional KV Cache Pools") as a selection
+ * rule on one HBM tier: the pools become the kept set, and the two metrics
+ * that decide the hot pool are applied per decode step.
+ *  (1) Temporal-aware pinning: the R = min(recent, lens[b]) most recent
+ *      tokens [len - R, len) are always kept.
+ *  (2) The older tokens [0, len - R) are ranked as in oracle_topk (key desc,
+ *      index asc) and the first min(k[b], len - R) are kept.
+ *  (3) Frequency-aware tracking: the hit-rate table hits[b][j] (2 bytes per
+ *      token, the table size Sec. 5.4 gives) counts the steps in which token
+ *      j was kept: +1 for every kept token, saturating at 65535.  hits may
+ *      be NULL.
+ * The kept set is emitted in ascending order, so the pinned window comes
+ * last.  If the window plus the ranked tokens exceed max_k, the window is cut
+ * to its max_k most recent tokens first, the ranked part gets what is left,
+ * and rc is 2.
+ */
+int oracle_bkp_select(int B, int cap, const int32_t* lens, const double* key, const int32_t* k,
+                      int recent, int max_k, int32_t* idx, int32_t* count, uint16_t* hits) {
+  int rc = 0;
+  if (recent < 0) recent = 0;
+  for (int b = 0; b < B; ++b) {
+    int len = lens[b] < cap ? lens[b] : cap;
+    if (len < 0) len = 0;
+    int R = recent < len ? recent : len;
+    int kb = k[b] < 0 ? 0 : k[b];
+    int n = kb < len - R ? kb : len - R;
+    if (R > max_k) {
+      R = max_k;
+      rc = 2;
+    }
+    if (n > max_k - R) {
+      n = max_k - R;
+      rc = 2;
+    }
+    const int older = len - (recent < len ? recent : len);   /* ranked range [0, older) */
+    or_item* items = (or_item*)malloc(sizeof(or_item) * (size_t)(older > 0 ? older : 1));
+    for (int j = 0; j < older; ++j) {
+      items[j].key = key[(int64_t)b * cap + j];
+      items[j].j = j;
+    }
+    qsort(items, (size_t)older, sizeof(or_item), or_cmp);
+    int32_t* row = idx + (int64_t)b * max_k;
+    for (int t = 0; t < n; ++t) row[t] = items[t].j;
+    qsort(row, (size_t)n, sizeof(int32_t), or_cmp_int);
+    for (int t = 0; t < R; ++t) row[n + t] = len - R + t;
+    for (int t = n + R; t < max_k; ++t) row[t] = -1;
+    count[b] = n + R;
+    if (hits)
+      for (int t = 0; t < n + R; ++t) {
+        uint16_t* hj = hits + (int64_t)b * cap + row[t];
+        if (*hj < 65535u) *hj = (uint16_t)(*hj + 1u);
+      }
+    free(items);
+  }
+  return rc;
+}
+
+/*
  * Step 5 -- attention of the current query over the selected tokens only
  * (Sec. 4.1, workflow step 6: only the critical KV is brought to the GPU for the
  * attention; Eq. 1 restricted to the selected set, the softmax renormalised

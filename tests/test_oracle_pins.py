@@ -224,6 +224,83 @@ def test_topk_nan_ranks_last(oracle_mod):
     assert idx[0, :3].tolist() == [1, 2, 4]
 
 
+# ---------------------------------------------------------------- BKP bookkeeping (Sec. 4.2)
+def test_bkp_without_window_is_topk(oracle_mod):
+    """recent = 0 reduces BKP selection to the pinned top-k, and the hit table
+    gains exactly one count at every kept token."""
+    rng = np.random.default_rng(11)
+    key = np.round(rng.standard_normal((5, 40)), 1)
+    lens, k = [40, 33, 1, 0, 25], [7, 33, 4, 2, 0]
+    hits0 = rng.integers(0, 50, size=(5, 40)).astype(np.uint16)
+    idx, count, rc, hits = oracle_mod.bkp_select(key, lens, k, 0, 40, hits0)
+    idx2, count2, rc2 = oracle_mod.topk(key, lens, k, 40)
+    assert rc == rc2 == 0 and np.array_equal(idx, idx2) and np.array_equal(count, count2)
+    want = hits0.astype(np.int64)
+    for b in range(5):
+        want[b, idx[b, : count[b]]] += 1
+    assert np.array_equal(hits.astype(np.int64), want)
+
+
+def test_bkp_window_and_exchange_property(oracle_mod):
+    """The kept set is the pinned window [len-R, len) plus a ranked set T of
+    min(k, len-R) older tokens such that no older token outside T beats one
+    inside it in (key desc, index asc) -- checked pair by pair, which fixes T
+    uniquely without sorting."""
+    rng = np.random.default_rng(12)
+    for trial in range(60):
+        cap = int(rng.integers(1, 14))
+        key = np.round(rng.standard_normal((1, cap)) * 2) / 2        # many ties
+        ln = int(rng.integers(0, cap + 1))
+        R_req = int(rng.integers(0, cap + 3))
+        kb = int(rng.integers(0, cap + 3))
+        idx, count, rc, _ = oracle_mod.bkp_select(key, [ln], [kb], R_req, cap + 4)
+        assert rc == 0
+        R = min(R_req, ln)
+        older = ln - R
+        got = idx[0, : count[0]].tolist()
+        assert got == sorted(got) and np.all(idx[0, count[0]:] == -1)
+        assert count[0] == R + min(kb, older)
+        assert got[len(got) - R:] == list(range(older, ln))          # the window, last
+        T = set(got[: len(got) - R])
+        assert all(j < older for j in T)
+        for i in T:
+            for j in range(older):
+                if j not in T:
+                    assert key[0, i] > key[0, j] or (key[0, i] == key[0, j] and i < j)
+
+
+def test_bkp_hits_count_steps_and_saturate(oracle_mod):
+    """Over several decode steps the table counts, per token, the steps that
+    kept it (tallied from the returned index sets), and stops at 65535."""
+    rng = np.random.default_rng(13)
+    cap, steps = 30, 9
+    hits = np.zeros((2, cap), dtype=np.uint16)
+    tally = np.zeros((2, cap), dtype=np.int64)
+    for t in range(steps):
+        key = rng.standard_normal((2, cap))
+        lens = [20 + t, 12 + t]
+        idx, count, rc, hits = oracle_mod.bkp_select(key, lens, [5, 3], 4, 16, hits)
+        assert rc == 0
+        for b in range(2):
+            tally[b, idx[b, : count[b]]] += 1
+    assert np.array_equal(hits.astype(np.int64), tally)
+    full = np.full((1, 6), 65534, dtype=np.uint16)
+    for _ in range(3):
+        _, _, _, full = oracle_mod.bkp_select(np.zeros((1, 6)), [6], [6], 0, 6, full)
+    assert np.all(full == 65535)
+
+
+def test_bkp_budget_cap_keeps_most_recent(oracle_mod):
+    """A window wider than max_k keeps its most recent tokens; otherwise the
+    ranked part gets what the window leaves; both report rc 2."""
+    key = np.arange(10, dtype=np.float64)[None, :]
+    idx, count, rc, _ = oracle_mod.bkp_select(key, [10], [3], 6, 4)
+    assert rc == 2 and count[0] == 4 and idx[0].tolist() == [6, 7, 8, 9]
+    # window [8, 9] first, then the best 2 of the older tokens: 6 and 7
+    idx, count, rc, _ = oracle_mod.bkp_select(key, [10], [3], 2, 4)
+    assert rc == 2 and idx[0].tolist() == [6, 7, 8, 9]
+
+
 def test_cec_single_head_raw_equals_attn_selection(oracle_mod):
     """Sec. 4.4: for one head and one step, ranking by raw q.K equals ranking by
     softmax weight (softmax is monotonic), so both modes select the same set."""
