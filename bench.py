@@ -232,6 +232,9 @@ def run_ours(args):
     w, lres = workload_for(args.workload, replica_seed(args.seed, rank), args.layers_resident)
     L, S, B, Hq, Hkv, d = w.layers, w.steps, w.batch, w.heads, w.kv_heads, w.head_dim
     cap, max_k = w.capacity, w.max_k
+    bkp = args.bkp_recent >= 0
+    if bkp:
+        max_k += args.bkp_recent   # the pinned window comes on top of the ranked budget
 
     # ---------------- resident inputs: caches, queries, lengths, budgets
     t_gen = time.time()
@@ -260,12 +263,21 @@ def run_ours(args):
     ws = hill.alloc_workspace(desc, mode, max_k, dev)
     stream = torch.cuda.Stream(device=dev)
 
+    hits = torch.zeros(lres, B, cap, dtype=torch.int16, device=dev) if bkp else None
+
+    def evict(t, l, o, st):
+        r = l % lres
+        acc = accum[r] if accum is not None else None
+        if bkp:
+            hill.hill_evict_step_bkp(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], args.bkp_recent,
+                                     max_k, mode, acc, scores[l], idx[l], count[l], hits[r], o, ws, st)
+        else:
+            hill.hill_evict_step(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], max_k, mode, acc,
+                                 scores[l], idx[l], count[l], o, ws, st)
+
     def issue_step(t, st):
         for l in range(L):
-            r = l % lres
-            hill.hill_evict_step(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], max_k, mode,
-                                 accum[r] if accum is not None else None, scores[l], idx[l], count[l],
-                                 out[l], ws, st)
+            evict(t, l, out[l], st)
 
     # eager warm-up of every kernel shape, then one CUDA graph per decode step
     with torch.cuda.stream(stream):
@@ -321,10 +333,7 @@ def run_ours(args):
     # with out = NULL, one graph per decode step, timed like the main region
     def issue_eval(t, st):
         for l in range(L):
-            r = l % lres
-            hill.hill_evict_step(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], max_k, mode,
-                                 accum[r] if accum is not None else None, scores[l], idx[l], count[l],
-                                 None, ws, st)
+            evict(t, l, None, st)
 
     eval_graphs = []
     for t in range(S):
@@ -405,7 +414,8 @@ def run_ours(args):
             "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(ms / len(order), 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f16" if w.dtype == torch.float16 else "bf16",
-            "data": "synthetic", "config": describe(w, lres, args.mode),
+            "data": "synthetic", "config": dict(describe(w, lres, args.mode),
+                                                **({"bkp_recent": args.bkp_recent} if bkp else {})),
             "k_stream_gbs": round(k_gbs, 1),
             "k_stream_frac_of_measured_hbm": round(k_gbs / world / peak, 4),
             "k_stream_frac_of_8tbs": round(k_gbs / world / 8000.0, 4),
@@ -576,6 +586,9 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--bkp-recent", type=int, default=-1,
+                    help="BKP bookkeeping (Sec. 4.2): pin this many recent tokens and keep a hit-rate table "
+                         "(hill_evict_step_bkp); default off")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         ap.error("--warmup must be at least 3")

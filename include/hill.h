@@ -125,6 +125,34 @@ hill_status hill_evict_step(const hill_desc* desc, const void* q, const void* k_
                             int32_t* idx, int32_t* count, float* out, void* ws,
                             size_t ws_bytes, void* stream);
 
+/* BKP bookkeeping (Sec. 4.2, Bidirectional KV Cache Pools), applied to the
+ * kept set of one HBM tier.  Two metrics decide which tokens stay:
+ *  - temporal-aware pinning: the W = min(recent, lens[b]) most recent tokens
+ *    [lens[b] - W, lens[b]) are always kept;
+ *  - the older tokens [0, lens[b] - W) are ranked as in hill_topk_select and
+ *    the first min(k[b], lens[b] - W) of them are kept;
+ *  - frequency-aware tracking: hits (nullable, [B][cap] uint16, caller-
+ *    owned and persistent across steps; the paper's 2-byte-per-token hit-rate
+ *    table) gains +1, saturating at 65535, at every kept token.
+ * idx[b] lists the kept tokens in ascending order (the window last), count[b]
+ * = kept tokens.  If the window plus the ranked tokens exceed max_k, the
+ * window keeps its max_k most recent tokens, the ranked part gets what is
+ * left, and HILL_ERR_DEVICE is recorded.  recent < 0 is HILL_ERR_INVALID_ARG;
+ * recent = 0 with hits = NULL is exactly hill_topk_select. */
+hill_status hill_topk_select_bkp(const hill_desc* desc, const float* scores, const int32_t* lens,
+                                 const int32_t* k, int32_t recent, int32_t max_k, int32_t* idx,
+                                 int32_t* count, uint16_t* hits, void* ws, size_t ws_bytes,
+                                 void* stream);
+
+/* hill_evict_step with the BKP selection of hill_topk_select_bkp in place of
+ * the plain top-k (same other arguments; recent = 0 with hits = NULL is
+ * exactly hill_evict_step). */
+hill_status hill_evict_step_bkp(const hill_desc* desc, const void* q, const void* k_cache,
+                                const void* v_cache, const int32_t* lens, const int32_t* k,
+                                int32_t recent, int32_t max_k, hill_score_mode mode, float* accum,
+                                float* scores, int32_t* idx, int32_t* count, uint16_t* hits, float* out,
+                                void* ws, size_t ws_bytes, void* stream);
+
 /* Synchronises `stream`, then returns and clears the device error word of the
  * current device: HILL_ERR_TIMEOUT if a bounded wait expired, HILL_ERR_DEVICE
  * if a device-side argument check fired, HILL_ERR_CUDA if the synchronisation

@@ -183,7 +183,7 @@ hill_status from_cuda(cudaError_t e) { return e == cudaSuccess ? HILL_OK : HILL_
 
 hill_status run_score(const hill_desc* d, const void* q, const void* k, const int32_t* lens, int mode,
                       float* scores, float* accum, unsigned char* base, const Layout& L,
-                      const DeviceInfo& di, cudaStream_t st, uint32_t* hist0 = nullptr) {
+                      const DeviceInfo& di, cudaStream_t st, uint32_t* hist0 = nullptr, int recent = 0) {
   if (d->batch == 0 || d->capacity == 0) return HILL_OK;
   const int G = d->num_q_heads / d->num_kv_heads;
   ScoreArgs a{};
@@ -226,12 +226,13 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   f.scores = scores;
   f.accum = accum;
   f.hist0 = hist0;
+  f.recent = recent;
   return from_cuda(counted(launch_attn_finalize(f, st), 1));
 }
 
 hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens, const int32_t* k,
                        int max_k, int32_t* idx, int32_t* count, const DeviceInfo& di, cudaStream_t st,
-                       const uint32_t* hist0 = nullptr) {
+                       const uint32_t* hist0 = nullptr, int recent = 0, uint16_t* hits = nullptr) {
   if (d->batch == 0) return HILL_OK;
   SelectArgs a{};
   a.key = key;
@@ -243,6 +244,8 @@ hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens
   a.idx = idx;
   a.count = count;
   a.hist0 = hist0;
+  a.recent = recent;
+  a.hits = hits;
   a.err = di.err;
   return from_cuda(counted(launch_select(a, st), 1));
 }
@@ -357,14 +360,15 @@ hill_status hill_gather_sparse_attn(const hill_desc* desc, const void* q, const 
                   static_cast<cudaStream_t>(stream));
 }
 
-hill_status hill_evict_step(const hill_desc* desc, const void* q, const void* k_cache, const void* v_cache,
-                            const int32_t* lens, const int32_t* k, int32_t max_k, hill_score_mode mode,
-                            float* accum, float* scores, int32_t* idx, int32_t* count, float* out, void* ws,
-                            size_t ws_bytes, void* stream) {
+static hill_status evict_step(const hill_desc* desc, const void* q, const void* k_cache, const void* v_cache,
+                              const int32_t* lens, const int32_t* k, int32_t recent, int32_t max_k,
+                              hill_score_mode mode, float* accum, float* scores, int32_t* idx, int32_t* count,
+                              uint16_t* hits, float* out, void* ws, size_t ws_bytes, void* stream) {
   hill_status s = check_desc(desc);
   if (s != HILL_OK) return s;
   if (mode != HILL_SCORE_ATTN && mode != HILL_SCORE_RAW) return HILL_ERR_INVALID_ARG;
-  if (max_k < 0 || !q || !k_cache || !lens || !k || !count || (max_k > 0 && !idx)) return HILL_ERR_INVALID_ARG;
+  if (max_k < 0 || recent < 0 || !q || !k_cache || !lens || !k || !count || (max_k > 0 && !idx))
+    return HILL_ERR_INVALID_ARG;
   if (out && !v_cache) return HILL_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(k_cache) || (out && !aligned16(v_cache))) return HILL_ERR_INVALID_ARG;
   DeviceInfo di;
@@ -376,12 +380,43 @@ hill_status hill_evict_step(const hill_desc* desc, const void* q, const void* k_
   float* s_out = scores ? scores : (accum ? nullptr : reinterpret_cast<float*>(base + L.scores));
   // ATTN: the normalisation also counts the leading key digit for the selection
   uint32_t* hist0 = L.has_hist0 ? reinterpret_cast<uint32_t*>(base + L.hist0) : nullptr;
-  s = run_score(desc, q, k_cache, lens, mode, s_out, accum, base, L, di, st, hist0);
+  s = run_score(desc, q, k_cache, lens, mode, s_out, accum, base, L, di, st, hist0, recent);
   if (s != HILL_OK) return s;
   const float* key = accum ? accum : s_out;
-  s = run_select(desc, key, lens, k, max_k, idx, count, di, st, hist0);
+  s = run_select(desc, key, lens, k, max_k, idx, count, di, st, hist0, recent, hits);
   if (s != HILL_OK || !out) return s;
   return run_attn(desc, q, k_cache, v_cache, idx, count, max_k, out, base, L, di, st);
+}
+
+hill_status hill_evict_step(const hill_desc* desc, const void* q, const void* k_cache, const void* v_cache,
+                            const int32_t* lens, const int32_t* k, int32_t max_k, hill_score_mode mode,
+                            float* accum, float* scores, int32_t* idx, int32_t* count, float* out, void* ws,
+                            size_t ws_bytes, void* stream) {
+  return evict_step(desc, q, k_cache, v_cache, lens, k, 0, max_k, mode, accum, scores, idx, count, nullptr, out,
+                    ws, ws_bytes, stream);
+}
+
+hill_status hill_evict_step_bkp(const hill_desc* desc, const void* q, const void* k_cache, const void* v_cache,
+                                const int32_t* lens, const int32_t* k, int32_t recent, int32_t max_k,
+                                hill_score_mode mode, float* accum, float* scores, int32_t* idx, int32_t* count,
+                                uint16_t* hits, float* out, void* ws, size_t ws_bytes, void* stream) {
+  return evict_step(desc, q, k_cache, v_cache, lens, k, recent, max_k, mode, accum, scores, idx, count, hits, out,
+                    ws, ws_bytes, stream);
+}
+
+hill_status hill_topk_select_bkp(const hill_desc* desc, const float* scores, const int32_t* lens,
+                                 const int32_t* k, int32_t recent, int32_t max_k, int32_t* idx, int32_t* count,
+                                 uint16_t* hits, void* ws, size_t ws_bytes, void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  hill_status s = check_desc(desc);
+  if (s != HILL_OK) return s;
+  if (max_k < 0 || recent < 0 || !scores || !lens || !k || !count || (max_k > 0 && !idx))
+    return HILL_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  return run_select(desc, scores, lens, k, max_k, idx, count, di, static_cast<cudaStream_t>(stream), nullptr,
+                    recent, hits);
 }
 
 hill_status hill_sync_status(void* stream) {

@@ -37,6 +37,7 @@ struct FinalizeArgs {
   float* scores;      // may be NULL when accum is given
   float* accum;       // may be NULL
   uint32_t* hist0;    // optional [B][2048]: counts of the leading 11-bit digit of the selection key
+  int recent;         // tokens j >= len - min(recent, len) are left out of hist0 (pinned, not ranked)
 };
 
 struct SelectArgs {
@@ -45,7 +46,9 @@ struct SelectArgs {
   const int32_t* k;
   int B, cap, max_k;
   int chunk;          // filled by the launcher
-  const uint32_t* hist0;   // optional [B][2048]: counts of the leading 11-bit key digit
+  const uint32_t* hist0;   // optional [B][2048]: counts of the leading 11-bit key digit (tokens j < len - recent)
+  int recent;         // BKP: the most recent min(recent, len) tokens are kept outright (0: none)
+  uint16_t* hits;     // BKP: optional [B][cap] hit-rate table, +1 (saturating) per kept token
   int32_t* idx;
   int32_t* count;
   unsigned* err;

@@ -450,7 +450,7 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
       key = a.accum[o] + s;
       a.accum[o] = key;
     }
-    if (a.hist0) atomicAdd(&hcount[ordered_key(key) >> 21], 1u);
+    if (a.hist0 && j < len - min(a.recent, len)) atomicAdd(&hcount[ordered_key(key) >> 21], 1u);
   }
   if (a.hist0) {
     __syncthreads();

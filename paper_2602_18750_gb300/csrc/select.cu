@@ -80,21 +80,39 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
 
   int len = a.lens[b];
   len = len < 0 ? 0 : (len > a.cap ? a.cap : len);
+  // BKP temporal pinning (Sec. 4.2): the most recent tokens [older, len) are
+  // kept outright; the ranking runs over [0, older)
+  const int rec = a.recent > 0 ? a.recent : 0;
+  const int rfull = rec < len ? rec : len;
+  const int older = len - rfull;
+  int win = rfull;
   int kk = a.k[b];
-  kk = kk < 0 ? 0 : (kk > len ? len : kk);
-  if (kk > a.max_k) {
+  kk = kk < 0 ? 0 : (kk > older ? older : kk);
+  if (win > a.max_k || kk > a.max_k - min(win, a.max_k)) {
     if (r == 0 && tid == 0) raise_error(a.err, kErrDevArg);
-    kk = a.max_k;
+    win = min(win, a.max_k);           // the most recent max_k tokens of the window
+    kk = min(kk, a.max_k - win);
   }
   int32_t* out = a.idx + (int64_t)b * a.max_k;
-  const int n = max(0, min(j_lo + a.chunk, len) - j_lo);
+  uint16_t* hits = a.hits ? a.hits + (int64_t)b * a.cap : nullptr;
+  auto hit = [&](int j) {   // the hit-rate table: +1 per kept token, saturating
+    if (hits && hits[j] != 0xffffu) hits[j] = (uint16_t)(hits[j] + 1u);
+  };
+  const int n = max(0, min(j_lo + a.chunk, older) - j_lo);
 
-  // padding and count (every path)
-  for (int p = kk + r * kSelThreads + tid; p < a.max_k; p += C * kSelThreads) out[p] = -1;
-  if (r == 0 && tid == 0) a.count[b] = kk;
+  // padding, count and the pinned window (every path)
+  for (int p = kk + win + r * kSelThreads + tid; p < a.max_k; p += C * kSelThreads) out[p] = -1;
+  if (r == 0 && tid == 0) a.count[b] = kk + win;
+  for (int j = max(j_lo, len - win) + tid; j < min(j_lo + a.chunk, len); j += kSelThreads) {
+    out[kk + j - (len - win)] = j;
+    hit(j);
+  }
   if (kk == 0) return;
-  if (kk == len) {  // everything is selected
-    for (int i = tid; i < n; i += kSelThreads) out[j_lo + i] = j_lo + i;
+  if (kk == older) {  // every older token is selected
+    for (int i = tid; i < n; i += kSelThreads) {
+      out[j_lo + i] = j_lo + i;
+      hit(j_lo + i);
+    }
     return;
   }
   __syncthreads();
@@ -243,8 +261,12 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
       ++eq_rank;
     }
     if (take) {
-      if (pos < (uint32_t)kk) out[pos] = j_lo + i;
-      else raise_error(a.err, kErrDevArg);   // cannot happen: more picks than the budget
+      if (pos < (uint32_t)kk) {
+        out[pos] = j_lo + i;
+        hit(j_lo + i);
+      } else {
+        raise_error(a.err, kErrDevArg);   // cannot happen: more picks than the budget
+      }
       ++pos;
     }
   }

@@ -7,7 +7,8 @@ libhill.so; there is no other implementation behind these names, and loading
 fails loudly if the library has not been built.
 
 Names follow the C ABI: :func:`hill_score`, :func:`hill_topk_select`,
-:func:`hill_gather_sparse_attn`, :func:`hill_evict_step`,
+:func:`hill_gather_sparse_attn`, :func:`hill_evict_step`, :func:`hill_topk_select_bkp`,
+:func:`hill_evict_step_bkp`,
 :func:`hill_workspace_bytes`, :func:`hill_sync_status`.
 """
 from __future__ import annotations
@@ -70,6 +71,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_topk_select.argtypes = [D, P, P, P, I32, P, P, P, SZ, P]
     lib.hill_gather_sparse_attn.argtypes = [D, P, P, P, P, P, I32, P, P, SZ, P]
     lib.hill_evict_step.argtypes = [D, P, P, P, P, P, I32, I32, P, P, P, P, P, P, SZ, P]
+    lib.hill_topk_select_bkp.argtypes = [D, P, P, P, I32, I32, P, P, P, P, SZ, P]
+    lib.hill_evict_step_bkp.argtypes = [D, P, P, P, P, P, I32, I32, I32, P, P, P, P, P, P, P, SZ, P]
     lib.hill_score_noalloc.argtypes = [D, P, P, P, I32, P, P, P]
     lib.hill_score_noalloc.restype = I32
     lib.hill_sync_status.argtypes = [P]
@@ -78,7 +81,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_abi_version.restype = I32
     lib.hill_kernel_launches.restype = ctypes.c_uint64
     for name in ("hill_score", "hill_topk_select", "hill_gather_sparse_attn", "hill_evict_step",
-                 "hill_sync_status"):
+                 "hill_topk_select_bkp", "hill_evict_step_bkp", "hill_sync_status"):
         getattr(lib, name).restype = I32
     _lib = lib
     return lib
@@ -180,6 +183,25 @@ def hill_evict_step(desc, q, k_cache, v_cache, lens, k, max_k, mode, accum, scor
     _check(load().hill_evict_step(ctypes.byref(desc), _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(lens),
                                   _ptr(k), int(max_k), int(mode), _ptr(accum), _ptr(scores), _ptr(idx),
                                   _ptr(count), _ptr(out), wp, wn, _stream(stream)), "hill_evict_step")
+
+
+def hill_topk_select_bkp(desc, scores, lens, k, recent, max_k, idx, count, hits=None, ws=None,
+                         stream=None) -> None:
+    """BKP selection (Sec. 4.2): the `recent` newest tokens pinned, the top-k of
+    the older ones, and hits[b][j] += 1 (saturating uint16) for kept tokens."""
+    wp, wn = _ws(ws)
+    _check(load().hill_topk_select_bkp(ctypes.byref(desc), _ptr(scores), _ptr(lens), _ptr(k), int(recent),
+                                       int(max_k), _ptr(idx), _ptr(count), _ptr(hits), wp, wn,
+                                       _stream(stream)), "hill_topk_select_bkp")
+
+
+def hill_evict_step_bkp(desc, q, k_cache, v_cache, lens, k, recent, max_k, mode, accum, scores, idx, count,
+                        hits, out, ws, stream=None) -> None:
+    wp, wn = _ws(ws)
+    _check(load().hill_evict_step_bkp(ctypes.byref(desc), _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(lens),
+                                      _ptr(k), int(recent), int(max_k), int(mode), _ptr(accum), _ptr(scores),
+                                      _ptr(idx), _ptr(count), _ptr(hits), _ptr(out), wp, wn,
+                                      _stream(stream)), "hill_evict_step_bkp")
 
 
 def hill_kernel_launches() -> int:

@@ -29,6 +29,7 @@ def _declared():
 def test_header_declares_the_boundary():
     names = _declared()
     for n in ("hill_score", "hill_topk_select", "hill_gather_sparse_attn", "hill_evict_step",
+              "hill_topk_select_bkp", "hill_evict_step_bkp",
               "hill_workspace_bytes", "hill_sync_status", "hill_status_string", "hill_abi_version"):
         assert n in names
 
@@ -95,6 +96,11 @@ def test_host_validation_without_device(lib):
     assert lib.hill_gather_sparse_attn(ctypes.byref(d), FAKE, FAKE, None, FAKE, FAKE, 8, FAKE, None, 0,
                                        None) == INV
     assert lib.hill_workspace_bytes(ctypes.byref(_desc(head_dim=64)), 0, 8) == 0
+    # BKP: a negative window is rejected before any device work
+    assert lib.hill_topk_select_bkp(ctypes.byref(d), FAKE, FAKE, FAKE, -1, 8, FAKE, FAKE, None, None, 0,
+                                    None) == INV
+    assert lib.hill_evict_step_bkp(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, -1, 8, 0, None, None, FAKE,
+                                   FAKE, None, None, FAKE, 1 << 30, None) == INV
 
 
 def test_binding_fails_loudly_without_library():
