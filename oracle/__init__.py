@@ -10,6 +10,8 @@ The arithmetic lives in ``hill_oracle.c`` (plain C, float64 on the exact
 arrays into it.  Each wrapper names the part of the paper it follows:
 
 * :func:`logits`       -- Eq. 1 (Sec. 2.1), q.K^T / sqrt(d) over the whole cache
+* :func:`logits_q8`    -- the same from E4M3 operands (Sec. 4.4 asymmetric precision),
+                          with :func:`quantize_rows`, :func:`e4m3_encode`, :func:`e4m3_decode`
 * :func:`scores`       -- Sec. 4.1 (column sum of softmax weights, ATTN) and
                           Sec. 4.4 (raw inner product, RAW)
 * :func:`accumulate`   -- running importance across decode steps (Sec. 4.2)
@@ -81,6 +83,13 @@ def _load():
             lib.oracle_evict_step.argtypes = [I, I, I, I, I, I, I, P, P, P, P, P, I,
                                               P, P, P, P, P, P]
             lib.oracle_decode16_array.argtypes = [I, P, P, ctypes.c_int64]
+            lib.oracle_e4m3_decode_array.argtypes = [P, P, ctypes.c_int64]
+            lib.oracle_e4m3_decode_array.restype = None
+            lib.oracle_e4m3_encode_array.argtypes = [P, P, ctypes.c_int64]
+            lib.oracle_e4m3_encode_array.restype = None
+            lib.oracle_quantize_rows.argtypes = [I, ctypes.c_int64, I, P, P, P]
+            lib.oracle_quantize_rows.restype = None
+            lib.oracle_logits_q8.argtypes = [I, I, I, I, I, I, P, P, P, P, P]
             lib.oracle_decode16_array.restype = None
             lib.oracle_accumulate.restype = None
             lib.oracle_num_threads.restype = I
@@ -133,6 +142,51 @@ def decode16(x, dtype=None) -> np.ndarray:
     out = np.empty(bits.shape, dtype=np.float64)
     _load().oracle_decode16_array(code, _ptr(bits), _ptr(out), bits.size)
     return out
+
+
+def e4m3_decode(codes) -> np.ndarray:
+    """Exact float64 values of E4M3 codes (uint8)."""
+    c = np.ascontiguousarray(codes, dtype=np.uint8)
+    out = np.empty(c.shape, dtype=np.float64)
+    _load().oracle_e4m3_decode_array(_ptr(c), _ptr(out), c.size)
+    return out
+
+
+def e4m3_encode(x) -> np.ndarray:
+    """Nearest E4M3 codes of float32 values (ties to even, saturating at 448)."""
+    v = np.ascontiguousarray(x, dtype=np.float32)
+    out = np.empty(v.shape, dtype=np.uint8)
+    _load().oracle_e4m3_encode_array(_ptr(v), _ptr(out), v.size)
+    return out
+
+
+def quantize_rows(x, dtype=None):
+    """Rows of the last dimension of a 16-bit tensor -> (codes uint8, scale float32)."""
+    code = _dtype_code(x, dtype)
+    bits = _bits(x)
+    d = bits.shape[-1]
+    rows = bits.size // d
+    codes = np.empty(bits.shape, dtype=np.uint8)
+    scale = np.empty(bits.shape[:-1], dtype=np.float32)
+    _load().oracle_quantize_rows(code, rows, d, _ptr(bits), _ptr(codes), _ptr(scale))
+    return codes, scale
+
+
+def logits_q8(q, kcodes, kscale, lens, dtype=None) -> np.ndarray:
+    """z8[B][H][cap] (NaN where j >= lens[b]) from the 8-bit operands (Sec. 4.4)."""
+    code = _dtype_code(q, dtype)
+    qb = _bits(q)
+    kc = np.ascontiguousarray(kcodes, dtype=np.uint8)
+    ks = np.ascontiguousarray(kscale, dtype=np.float32)
+    B, H, d = qb.shape
+    _, Hkv, cap, d2 = kc.shape
+    assert d2 == d and ks.shape == (B, Hkv, cap)
+    z = np.full((B, H, cap), np.nan)
+    rc = _load().oracle_logits_q8(code, B, H, Hkv, d, cap, _ptr(qb), _ptr(kc), _ptr(ks), _ptr(_i32(lens)),
+                                  _ptr(z))
+    if rc:
+        raise ValueError(f"oracle_logits_q8 rc={rc}")
+    return z
 
 
 def logits(q, K, lens, dtype=None) -> np.ndarray:

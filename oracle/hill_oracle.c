@@ -111,6 +111,119 @@ int oracle_logits(int dtype, int B, int H, int Hkv, int d, int cap,
 }
 
 /*
+ * CEC asymmetric precision (Sec. 4.4): the evaluation may rank tokens with
+ * low-precision inner products while the attention keeps the original keys.
+ * Here the keys' shadow is OCP FP8 E4M3 with one scale per (b, g, j) row and
+ * the query is cast the same way per (b, h).
+ * E4M3: 1 sign bit, 4 exponent bits (bias 7), 3 fraction bits; exponent 0
+ * holds zero and the subnormals f * 2^-9; the largest finite magnitude is
+ * 1.75 * 2^8 = 448; S.1111.111 is NaN; there is no infinity.
+ */
+double oracle_e4m3_decode(uint8_t c) {
+  const int e = (c >> 3) & 15, f = c & 7;
+  if (e == 15 && f == 7) return NAN;
+  const double v = e == 0 ? ldexp((double)f, -9) : ldexp(1.0 + f / 8.0, e - 7);
+  return (c & 0x80) ? -v : v;
+}
+
+/* Nearest E4M3 value of a finite float, ties to the even code, magnitudes
+ * from 448 up saturating to 448. */
+uint8_t oracle_e4m3_encode(float xf) {
+  const double x = xf;
+  const uint8_t sign = signbit(x) ? 0x80 : 0x00;
+  const double a = fabs(x);
+  if (a >= 448.0) return sign | 0x7e;
+  if (a == 0.0) return sign;
+  int ex;
+  (void)frexp(a, &ex);                                   /* a = m * 2^ex, m in [0.5, 1) */
+  /* spacing of the representable values around a: 2^-9 below 2^-6, else
+   * 2^(floor(log2 a) - 3) */
+  const double qs = a < ldexp(1.0, -6) ? ldexp(1.0, -9) : ldexp(1.0, ex - 1 - 3);
+  const double n = a / qs;                               /* exact: qs is a power of two */
+  long k = (long)floor(n);
+  const double rem = n - (double)k;
+  if (rem > 0.5 || (rem == 0.5 && (k & 1))) k += 1;
+  const double v = (double)k * qs;                       /* at most 448 */
+  if (v < ldexp(1.0, -6)) return sign | (uint8_t)k;      /* subnormal: code = f */
+  int ev;
+  (void)frexp(v, &ev);
+  const int E = ev - 1 + 7;
+  const int f = (int)((ldexp(v, -(ev - 1)) - 1.0) * 8.0);
+  return sign | (uint8_t)(E << 3) | (uint8_t)f;
+}
+
+void oracle_e4m3_decode_array(const uint8_t* c, double* out, int64_t n) {
+  for (int64_t i = 0; i < n; ++i) out[i] = oracle_e4m3_decode(c[i]);
+}
+
+void oracle_e4m3_encode_array(const float* x, uint8_t* out, int64_t n) {
+  for (int64_t i = 0; i < n; ++i) out[i] = oracle_e4m3_encode(x[i]);
+}
+
+/* Quantise rows of d 16-bit values: amax = max_i |x_i| (exact), r = 448 /
+ * amax and y_i = x_i * r in float32 arithmetic, code_i = e4m3(y_i), scale =
+ * amax / 448 in float32 (so code_i * scale ~ x_i, the largest entry exactly
+ * 448 * scale).  An all-zero row gives zero codes and scale 0.  The float32
+ * steps are the ones the kernel takes, so both sides pick the same codes. */
+void oracle_quantize_rows(int dtype, int64_t rows, int d, const uint16_t* x, uint8_t* codes, float* scale) {
+  for (int64_t r = 0; r < rows; ++r) {
+    const uint16_t* xr = x + r * d;
+    float amax = 0.0f;
+    for (int i = 0; i < d; ++i) {
+      const float v = (float)fabs(oracle_decode16(dtype, xr[i]));
+      if (v > amax) amax = v;
+    }
+    uint8_t* cr = codes + r * d;
+    if (amax == 0.0f) {
+      for (int i = 0; i < d; ++i) cr[i] = 0;
+      scale[r] = 0.0f;
+      continue;
+    }
+    const volatile float inv = 448.0f / amax;
+    for (int i = 0; i < d; ++i) {
+      const volatile float y = (float)oracle_decode16(dtype, xr[i]) * inv;
+      cr[i] = oracle_e4m3_encode(y);
+    }
+    const volatile float sc = amax / 448.0f;
+    scale[r] = sc;
+  }
+}
+
+/*
+ * Logits from the 8-bit operands: q[b,h,:] is quantised like a key row
+ * (codes qc, scale sq) and
+ *   z8[b,h,j] = (sum_i e4m3(qc_i) * e4m3(kc[b,g,j,i])) * sq * sk[b,g,j] / sqrt(d)
+ * for j < lens[b]; kc [B][Hkv][cap][d] codes, sk [B][Hkv][cap] scales.
+ */
+int oracle_logits_q8(int dtype, int B, int H, int Hkv, int d, int cap, const uint16_t* q,
+                     const uint8_t* kc, const float* sk, const int32_t* lens, double* z) {
+  if (B < 0 || H <= 0 || Hkv <= 0 || H % Hkv || d <= 0 || cap < 0) return 1;
+  const int G = H / Hkv;
+  const double inv_sqrt_d = 1.0 / sqrt((double)d);
+  int bh;
+#pragma omp parallel for schedule(dynamic)
+  for (bh = 0; bh < B * H; ++bh) {
+    const int b = bh / H, h = bh % H, g = h / G;
+    const int len = lens[b] < cap ? lens[b] : cap;
+    uint8_t* qc = (uint8_t*)malloc((size_t)d);
+    float sq;
+    oracle_quantize_rows(dtype, 1, d, q + ((int64_t)b * H + h) * d, qc, &sq);
+    double* qv = (double*)malloc(sizeof(double) * (size_t)d);
+    for (int i = 0; i < d; ++i) qv[i] = oracle_e4m3_decode(qc[i]);
+    for (int j = 0; j < len; ++j) {
+      const int64_t row = ((int64_t)b * Hkv + g) * cap + j;
+      const uint8_t* kr = kc + row * d;
+      double acc = 0.0;
+      for (int i = 0; i < d; ++i) acc += qv[i] * oracle_e4m3_decode(kr[i]);
+      z[((int64_t)b * H + h) * cap + j] = acc * (double)sq * (double)sk[row] * inv_sqrt_d;
+    }
+    free(qv);
+    free(qc);
+  }
+  return 0;
+}
+
+/*
  * Step 2 -- per-token importance.
  *  ATTN (the paper's definition, Sec. 4.1 "System Workflow"): a token's
  *    importance is the column-wise sum of its attention weights.  The weights

@@ -224,6 +224,93 @@ def test_topk_nan_ranks_last(oracle_mod):
     assert idx[0, :3].tolist() == [1, 2, 4]
 
 
+# ---------------------------------------------------------------- E4M3 shadow (Sec. 4.4)
+def test_e4m3_decode_all_codes_matches_torch(oracle_mod):
+    codes = np.arange(256, dtype=np.uint8)
+    got = oracle_mod.e4m3_decode(codes)
+    ref = torch.from_numpy(codes).view(torch.float8_e4m3fn).double().numpy()
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(got), nan) and nan.sum() == 2
+    assert np.array_equal(got[~nan], ref[~nan])
+    assert got[0x7E] == 448.0 and got[0x01] == 2.0 ** -9 and got[0x08] == 2.0 ** -6
+
+
+def test_e4m3_encode_round_trip_ties_and_torch(oracle_mod):
+    codes = np.array([c for c in range(256) if (c & 0x7F) != 0x7F], dtype=np.uint8)
+    vals = oracle_mod.e4m3_decode(codes)
+    assert np.array_equal(oracle_mod.e4m3_encode(vals.astype(np.float32)), codes)     # round trip
+    pos = np.sort(np.unique(vals[vals > 0]))
+    mids = (pos[:-1] + pos[1:]) / 2                    # exact midpoints (float32-representable)
+    enc = oracle_mod.e4m3_encode(mids.astype(np.float32))
+    lo = oracle_mod.e4m3_encode(pos[:-1].astype(np.float32))
+    hi = oracle_mod.e4m3_encode(pos[1:].astype(np.float32))
+    assert np.all(enc == np.where(lo % 2 == 0, lo, hi))                            # ties to the even code
+    rng = np.random.default_rng(3)
+    x = np.concatenate([rng.uniform(-463, 463, 20000), rng.uniform(-0.02, 0.02, 20000),
+                        [448.0, -0.0]]).astype(np.float32)
+    ref = torch.from_numpy(x).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+    assert np.array_equal(oracle_mod.e4m3_encode(x), ref)
+    # beyond the last rounding interval torch's cast gives NaN; the encoder
+    # (like the kernel's saturating conversion) gives +-448
+    assert oracle_mod.e4m3_encode(np.array([500.0, -1e4, 3e38], np.float32)).tolist() == [0x7E, 0xFE, 0x7E]
+
+
+def test_quantize_rows_bounds(oracle_mod):
+    g = torch.Generator().manual_seed(4)
+    x = (torch.randn(64, 128, generator=g) * torch.logspace(-3, 2, 64)[:, None]).half()
+    x[5] = 0.0
+    codes, scale = oracle_mod.quantize_rows(x)
+    xd = oracle_mod.decode16(x)
+    amax = np.abs(xd).max(axis=1)
+    assert scale[5] == 0.0 and np.all(codes[5] == 0)
+    for r in range(64):
+        if r == 5:
+            continue
+        assert scale[r] == np.float32(np.float32(amax[r]) / np.float32(448.0))
+        dec = oracle_mod.e4m3_decode(codes[r])
+        y = xd[r] * np.float64(np.float32(448.0) / np.float32(amax[r]))
+        assert np.abs(dec).max() == 448.0
+        # E4M3 rounding error: half a spacing, i.e. 1/16 relative above 2^-6, 2^-10 below
+        assert np.all(np.abs(dec - y) <= np.maximum(np.abs(y) / 16, 2.0 ** -10) * (1 + 1e-6))
+
+
+def test_logits_q8_is_fp64_matmul_of_dequantized(oracle_mod):
+    B, H, Hkv, d, cap = 2, 8, 2, 128, 40
+    lens = [40, 23]
+    q, K, _, _ = inputs.random_case(B, H, Hkv, d, cap, lens, seed=8)
+    kc, ks = oracle_mod.quantize_rows(K)
+    qc, qs = oracle_mod.quantize_rows(q)
+    Kd = torch.from_numpy(oracle_mod.e4m3_decode(kc) * ks[..., None].astype(np.float64))
+    qd = torch.from_numpy(oracle_mod.e4m3_decode(qc) * qs[..., None].astype(np.float64))
+    ref = torch.matmul(_expand_kv(Kd, H), qd.unsqueeze(-1)).squeeze(-1) / math.sqrt(d)
+    z8 = oracle_mod.logits_q8(q, kc, ks, lens)
+    for b in range(B):
+        assert np.allclose(z8[b, :, : lens[b]], ref[b, :, : lens[b]].numpy(), rtol=1e-12, atol=1e-12)
+        assert np.all(np.isnan(z8[b, :, lens[b]:]))
+
+
+def test_logits_q8_lossless_rows_equal_exact_logits(oracle_mod):
+    """Rows built from E4M3 values times 2^-4 whose largest magnitude is 448 * 2^-4
+    quantise without loss, so the 8-bit logits equal the exact ones."""
+    rng = np.random.default_rng(9)
+    grid = oracle_mod.e4m3_decode(np.arange(0, 0x7F, dtype=np.uint8))
+    grid = grid[grid >= 2.0 ** -6]                     # normals: exact in binary16 after the 2^-4 shift
+    B, H, Hkv, d, cap = 1, 4, 2, 128, 17
+
+    def rows(n):
+        v = rng.choice(grid, size=(n, d)) * rng.choice([-1.0, 1.0], size=(n, d))
+        v[np.arange(n), rng.integers(0, d, n)] = 448.0
+        return torch.from_numpy(v * 2.0 ** -4).half()
+
+    q = rows(B * H).reshape(B, H, d)
+    K = rows(B * Hkv * cap).reshape(B, Hkv, cap, d)
+    kc, ks = oracle_mod.quantize_rows(K)
+    assert np.all(ks == np.float32(28.0 / 448.0))
+    z8 = oracle_mod.logits_q8(q, kc, ks, [cap])
+    z = oracle_mod.logits(q, K, [cap])
+    assert np.allclose(z8, z, rtol=1e-12, atol=0)
+
+
 # ---------------------------------------------------------------- BKP bookkeeping (Sec. 4.2)
 def test_bkp_without_window_is_topk(oracle_mod):
     """recent = 0 reduces BKP selection to the pinned top-k, and the hit table
