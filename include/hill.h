@@ -153,6 +153,40 @@ hill_status hill_evict_step_bkp(const hill_desc* desc, const void* q, const void
                                 float* scores, int32_t* idx, int32_t* count, uint16_t* hits, float* out,
                                 void* ws, size_t ws_bytes, void* stream);
 
+/* Asymmetric-precision scoring (Sec. 4.4, CEC): the evaluation ranks tokens
+ * with low-precision inner products, while the attention keeps the original
+ * 16-bit keys and values.  On this GPU the low precision is OCP FP8 E4M3
+ * (its tensor-core rate is ~14x that of INT8 here), one scale per key row:
+ *   k8     [B][Hkv][cap][128] uint8 E4M3 codes, dense, 16-byte aligned;
+ *   kscale [B][Hkv][cap32] float32, cap32 = cap rounded up to 32, dense.
+ * A row's codes are e4m3(K_i * (448 / amax)) with amax = max_i |K_i| (float32
+ * product, round to nearest even, saturating) and its scale is amax / 448.
+ * The query is cast the same way per (b, h) inside the scoring kernel, and
+ *   z8 = (sum_i e4m3(q)_i e4m3(K)_i) * s_q * s_k / sqrt(d)
+ * replaces the logit of Eq. 1 in the importance (ATTN or RAW, as hill_score).
+ *
+ * hill_quantize_k writes the shadow of rows [row_begin[b], row_end[b]) of
+ * every KV head (device arrays [B], clamped to [0, cap]); max_rows bounds
+ * row_end - row_begin over b (e.g. 1 to add this step's token, cap to build
+ * the whole shadow). */
+hill_status hill_quantize_k(const hill_desc* desc, const void* k_cache, const int32_t* row_begin,
+                            const int32_t* row_end, int32_t max_rows, uint8_t* k8, float* kscale,
+                            void* stream);
+
+/* hill_score on the E4M3 shadow (same outputs and workspace as hill_score). */
+hill_status hill_score_f8(const hill_desc* desc, const void* q, const uint8_t* k8, const float* kscale,
+                          const int32_t* lens, hill_score_mode mode, float* scores, float* accum,
+                          void* ws, size_t ws_bytes, void* stream);
+
+/* hill_evict_step with the scoring on the E4M3 shadow; the sparse attention
+ * (out != NULL) reads the original k_cache and v_cache.  k_cache and v_cache
+ * may be NULL when out is NULL. */
+hill_status hill_evict_step_f8(const hill_desc* desc, const void* q, const uint8_t* k8, const float* kscale,
+                               const void* k_cache, const void* v_cache, const int32_t* lens,
+                               const int32_t* k, int32_t max_k, hill_score_mode mode, float* accum,
+                               float* scores, int32_t* idx, int32_t* count, float* out, void* ws,
+                               size_t ws_bytes, void* stream);
+
 /* Synchronises `stream`, then returns and clears the device error word of the
  * current device: HILL_ERR_TIMEOUT if a bounded wait expired, HILL_ERR_DEVICE
  * if a device-side argument check fired, HILL_ERR_CUDA if the synchronisation

@@ -113,6 +113,27 @@ hill_status make_kmap(const hill_desc* d, const void* k, ScoreArgs* a) {
   return r == CUDA_SUCCESS ? HILL_OK : HILL_ERR_UNSUPPORTED;
 }
 
+// Tiled tensor map of the dense E4M3 key shadow [B][Hkv][cap][128] (one
+// byte per code): box = 128 codes (one 128-byte swizzled row) x 32 tokens.
+hill_status make_kmap8(const hill_desc* d, const void* k8, ScoreArgs* a) {
+  auto fn = encode_tiled();
+  if (!fn) return HILL_ERR_CUDA;
+  const cuuint64_t cap = (cuuint64_t)std::max(d->capacity, 1), hkv = (cuuint64_t)d->num_kv_heads;
+  cuuint64_t gdim[4] = {(cuuint64_t)kHeadDim, cap, hkv, (cuuint64_t)std::max(d->batch, 1)};
+  cuuint64_t gstr[3] = {(cuuint64_t)kHeadDim, cap * kHeadDim, hkv * cap * kHeadDim};
+  cuuint32_t box[4] = {(cuuint32_t)kHeadDim, 32, 1, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  a->kdim_tok = 1;
+  a->kdim_head = 2;
+  a->kdim_seq = 3;
+  CUresult r = fn(&a->kmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<void*>(k8), gdim, gstr, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? HILL_OK : HILL_ERR_UNSUPPORTED;
+}
+
+int cap32_of(const hill_desc* d) { return (d->capacity + 31) & ~31; }
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 bool stride_ok(int64_t s) { return s >= 0 && (s % 8) == 0; }
 
@@ -183,7 +204,8 @@ hill_status from_cuda(cudaError_t e) { return e == cudaSuccess ? HILL_OK : HILL_
 
 hill_status run_score(const hill_desc* d, const void* q, const void* k, const int32_t* lens, int mode,
                       float* scores, float* accum, unsigned char* base, const Layout& L,
-                      const DeviceInfo& di, cudaStream_t st, uint32_t* hist0 = nullptr, int recent = 0) {
+                      const DeviceInfo& di, cudaStream_t st, uint32_t* hist0 = nullptr, int recent = 0,
+                      const float* kscale = nullptr) {
   if (d->batch == 0 || d->capacity == 0) return HILL_OK;
   const int G = d->num_q_heads / d->num_kv_heads;
   ScoreArgs a{};
@@ -201,8 +223,12 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   a.k_sn = d->k_sn;
   a.nslot = L.score_grid;
   a.err = di.err;
-  hill_status ms = make_kmap(d, k, &a);
+  // kscale != NULL: k is the E4M3 shadow of the keys (asymmetric-precision scoring)
+  const bool f8 = kscale != nullptr;
+  hill_status ms = f8 ? make_kmap8(d, k, &a) : make_kmap(d, k, &a);
   if (ms != HILL_OK) return ms;
+  a.kscale = kscale;
+  a.cap32 = cap32_of(d);
   const bool raw = mode == HILL_SCORE_RAW;
   if (raw) {
     a.scores = scores;
@@ -213,7 +239,7 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
     a.hist0 = hist0;
     a.hist0_words = (int64_t)d->batch * select_hist_bins();
   }
-  hill_status s = from_cuda(counted(launch_score(a, d->dtype, G, raw, L.score_grid, st), 1));
+  hill_status s = from_cuda(counted(launch_score(a, d->dtype, G, raw, f8, L.score_grid, st), 1));
   if (s != HILL_OK || raw) return s;
   FinalizeArgs f{};
   f.logits = a.logits;
@@ -363,14 +389,16 @@ hill_status hill_gather_sparse_attn(const hill_desc* desc, const void* q, const 
 static hill_status evict_step(const hill_desc* desc, const void* q, const void* k_cache, const void* v_cache,
                               const int32_t* lens, const int32_t* k, int32_t recent, int32_t max_k,
                               hill_score_mode mode, float* accum, float* scores, int32_t* idx, int32_t* count,
-                              uint16_t* hits, float* out, void* ws, size_t ws_bytes, void* stream) {
+                              uint16_t* hits, float* out, void* ws, size_t ws_bytes, void* stream,
+                              const uint8_t* k8 = nullptr, const float* kscale = nullptr) {
   hill_status s = check_desc(desc);
   if (s != HILL_OK) return s;
   if (mode != HILL_SCORE_ATTN && mode != HILL_SCORE_RAW) return HILL_ERR_INVALID_ARG;
-  if (max_k < 0 || recent < 0 || !q || !k_cache || !lens || !k || !count || (max_k > 0 && !idx))
+  if (max_k < 0 || recent < 0 || !q || !lens || !k || !count || (max_k > 0 && !idx)) return HILL_ERR_INVALID_ARG;
+  if (k8 ? (!kscale || !aligned16(k8) || !aligned16(kscale)) : !k_cache) return HILL_ERR_INVALID_ARG;
+  if (out && (!k_cache || !v_cache)) return HILL_ERR_INVALID_ARG;
+  if (!aligned16(q) || (k_cache && !aligned16(k_cache)) || (out && !aligned16(v_cache)))
     return HILL_ERR_INVALID_ARG;
-  if (out && !v_cache) return HILL_ERR_INVALID_ARG;
-  if (!aligned16(q) || !aligned16(k_cache) || (out && !aligned16(v_cache))) return HILL_ERR_INVALID_ARG;
   DeviceInfo di;
   if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
   const Layout L = layout_for(desc, mode, max_k, di.sms);
@@ -380,7 +408,8 @@ static hill_status evict_step(const hill_desc* desc, const void* q, const void* 
   float* s_out = scores ? scores : (accum ? nullptr : reinterpret_cast<float*>(base + L.scores));
   // ATTN: the normalisation also counts the leading key digit for the selection
   uint32_t* hist0 = L.has_hist0 ? reinterpret_cast<uint32_t*>(base + L.hist0) : nullptr;
-  s = run_score(desc, q, k_cache, lens, mode, s_out, accum, base, L, di, st, hist0, recent);
+  s = run_score(desc, q, k8 ? static_cast<const void*>(k8) : k_cache, lens, mode, s_out, accum, base, L, di, st,
+                hist0, recent, kscale);
   if (s != HILL_OK) return s;
   const float* key = accum ? accum : s_out;
   s = run_select(desc, key, lens, k, max_k, idx, count, di, st, hist0, recent, hits);
@@ -417,6 +446,57 @@ hill_status hill_topk_select_bkp(const hill_desc* desc, const float* scores, con
   if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
   return run_select(desc, scores, lens, k, max_k, idx, count, di, static_cast<cudaStream_t>(stream), nullptr,
                     recent, hits);
+}
+
+hill_status hill_quantize_k(const hill_desc* desc, const void* k_cache, const int32_t* row_begin,
+                            const int32_t* row_end, int32_t max_rows, uint8_t* k8, float* kscale, void* stream) {
+  hill_status s = check_desc(desc);
+  if (s != HILL_OK) return s;
+  if (!k_cache || !row_begin || !row_end || !k8 || !kscale || max_rows < 0) return HILL_ERR_INVALID_ARG;
+  if (!aligned16(k_cache) || !aligned16(k8) || !aligned16(kscale)) return HILL_ERR_INVALID_ARG;
+  if (desc->batch == 0 || desc->capacity == 0 || max_rows == 0) return HILL_OK;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  QuantArgs a{};
+  a.k = k_cache;
+  a.row_begin = row_begin;
+  a.row_end = row_end;
+  a.B = desc->batch;
+  a.Hkv = desc->num_kv_heads;
+  a.cap = desc->capacity;
+  a.cap32 = cap32_of(desc);
+  a.k_sb = desc->k_sb;
+  a.k_sh = desc->k_sh;
+  a.k_sn = desc->k_sn;
+  a.k8 = k8;
+  a.kscale = kscale;
+  return from_cuda(counted(launch_quantize_k(a, desc->dtype, std::min(max_rows, desc->capacity),
+                                             static_cast<cudaStream_t>(stream)), 1));
+}
+
+hill_status hill_score_f8(const hill_desc* desc, const void* q, const uint8_t* k8, const float* kscale,
+                          const int32_t* lens, hill_score_mode mode, float* scores, float* accum, void* ws,
+                          size_t ws_bytes, void* stream) {
+  hill_status s = check_desc(desc);
+  if (s != HILL_OK) return s;
+  if (mode != HILL_SCORE_ATTN && mode != HILL_SCORE_RAW) return HILL_ERR_INVALID_ARG;
+  if (!q || !k8 || !kscale || !lens || !scores) return HILL_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k8) || !aligned16(kscale)) return HILL_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  const Layout L = layout_for(desc, mode, 0, di.sms);
+  if (!ws || ws_bytes < L.total) return HILL_ERR_WORKSPACE;
+  return run_score(desc, q, k8, lens, mode, scores, accum, ws_base(ws), L, di, static_cast<cudaStream_t>(stream),
+                   nullptr, 0, kscale);
+}
+
+hill_status hill_evict_step_f8(const hill_desc* desc, const void* q, const uint8_t* k8, const float* kscale,
+                               const void* k_cache, const void* v_cache, const int32_t* lens, const int32_t* k,
+                               int32_t max_k, hill_score_mode mode, float* accum, float* scores, int32_t* idx,
+                               int32_t* count, float* out, void* ws, size_t ws_bytes, void* stream) {
+  if (!k8 || !kscale) return HILL_ERR_INVALID_ARG;
+  return evict_step(desc, q, k_cache, v_cache, lens, k, 0, max_k, mode, accum, scores, idx, count, nullptr, out,
+                    ws, ws_bytes, stream, k8, kscale);
 }
 
 hill_status hill_sync_status(void* stream) {

@@ -209,6 +209,24 @@ __device__ __forceinline__ uint32_t lds32(uint32_t addr) {
 
 // D += A (16x16, row) * B (16x8, col) with fp32 accumulation; A and B share
 // the element type (fp16 for DT 0, bf16 for DT 1).
+// D += A . B on E4M3 operands (m16n8k32, fp32 accumulation): A row-major
+// 16x32, B column-major 32x8, four E4M3 codes per 32-bit register.
+__device__ __forceinline__ void mma_16832_e4m3(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k32.row.col.f32.e4m3.e4m3.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Two floats -> two E4M3 codes in one 16-bit value (x in the low byte),
+// rounded to nearest even, magnitudes beyond 448 saturating to 448.
+__device__ __forceinline__ uint32_t e4m3x2(float x, float y) {
+  unsigned short v;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(v) : "f"(y), "f"(x));
+  return v;
+}
+
 template <int DT>
 __device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1);
 

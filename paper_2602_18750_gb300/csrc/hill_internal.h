@@ -13,6 +13,9 @@ namespace hill {
 
 struct ScoreArgs {
   CUtensorMap kmap;   // K cache: 4-D tiled map, 128-byte swizzle, box = 64 dims x kT tokens
+                      // (E4M3 shadow: box = 128 codes x kT tokens)
+  const float* kscale;   // E4M3 shadow: [B][Hkv][cap32] row scales
+  int cap32;
   int kdim_tok, kdim_head, kdim_seq;   // which tensor-map dimension holds token, KV head, sequence
   const void* q;
   const void* k;
@@ -38,6 +41,16 @@ struct FinalizeArgs {
   float* accum;       // may be NULL
   uint32_t* hist0;    // optional [B][2048]: counts of the leading 11-bit digit of the selection key
   int recent;         // tokens j >= len - min(recent, len) are left out of hist0 (pinned, not ranked)
+};
+
+struct QuantArgs {
+  const void* k;              // 16-bit K cache, strides k_sb, k_sh, k_sn
+  const int32_t* row_begin;   // [B] rows [row_begin[b], row_end[b]) are quantised
+  const int32_t* row_end;
+  int B, Hkv, cap, cap32;     // cap32 = cap rounded up to 32 (row length of kscale)
+  int64_t k_sb, k_sh, k_sn;
+  uint8_t* k8;                // [B][Hkv][cap][128] E4M3 codes
+  float* kscale;              // [B][Hkv][cap32]
 };
 
 struct SelectArgs {
@@ -115,13 +128,16 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
 }
 
 // score.cu
-size_t score_smem_bytes(int G);
+size_t score_smem_bytes(int G, bool f8);
 int score_tile_tokens();
 int score_warps();
 int score_max_batch();
 int score_max_kv_heads(int G);
-cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, int grid, cudaStream_t st);
+cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8, int grid, cudaStream_t st);
 cudaError_t launch_attn_finalize(const FinalizeArgs& a, cudaStream_t st);
+
+// quant.cu
+cudaError_t launch_quantize_k(const QuantArgs& a, int dtype, int max_rows, cudaStream_t st);
 
 // select.cu
 int select_cluster_size(int cap);

@@ -40,13 +40,15 @@ constexpr int kMaxNg = 4;                   // KV heads per warp per item (Hkv <
 constexpr int kBoxBytes = kT * 128;         // one 64-dim half of a tile: 32 swizzled 128-byte rows
 constexpr int kKBytes = 2 * kBoxBytes;
 
-template <int G>
+template <int G, bool F8>
 struct ScoreCfg {
-  static constexpr int kSlotBytes = kKBytes;               // one K tile (a multiple of 1024)
-  static constexpr int kSW = 3;                            // stages per warp
+  // one K tile (a multiple of 1024): 8 KB of 16-bit keys, or 4 KB of E4M3 codes
+  static constexpr int kSlotBytes = F8 ? kT * 128 : kKBytes;
+  static constexpr int kSW = F8 ? 6 : 3;                   // stages per warp (same bytes in flight)
   static constexpr int kStages = kNW * kSW;
   // shared-memory layout (offsets from a 1024-byte aligned base)
-  static constexpr int kOffBar = kStages * kSlotBytes;
+  static constexpr int kOffScale = kStages * kSlotBytes;   // F8: the kT token scales of each stage
+  static constexpr int kOffBar = kOffScale + (F8 ? kStages * kT * 4 : 0);
   static constexpr int kOffTab = kOffBar + kStages * 8;
   static constexpr int kOffRed = kOffTab + 2 * kTableInts * 4;
   static constexpr int kOffFlag = kOffRed + 2 * kNW * kT * 4;
@@ -73,9 +75,9 @@ struct Cursor {
   int item, r, b;
 };
 
-template <int DT, int G, bool RAW>
+template <int DT, int G, bool RAW, bool F8>
 __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_constant__ ScoreArgs a) {
-  using Cfg = ScoreCfg<G>;
+  using Cfg = ScoreCfg<G, F8>;
   constexpr int kSlotBytes = Cfg::kSlotBytes;
   constexpr int kSW = Cfg::kSW;
   constexpr int kStages = Cfg::kStages;
@@ -135,6 +137,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   const uint64_t pol = l2_evict_first_policy();
   const uint32_t stage0 = base_addr + warp * kSW * kSlotBytes;
   const uint32_t bar0 = base_addr + Cfg::kOffBar + warp * kSW * 8;
+  const uint32_t scale0 = base_addr + Cfg::kOffScale + warp * kSW * kT * 4;   // F8 only
   const int b_first = find_seq(tstart, B, blockIdx.x);
 
   auto advance = [&](Cursor& c) {
@@ -150,13 +153,20 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
     const int g = warp + c.r * kNW;
     const uint32_t fb = bar0 + s * 8;
     const uint32_t dst = stage0 + s * kSlotBytes;
-    mbar_arrive_expect_tx(fb, (uint32_t)kKBytes);
     // tensor-map coordinates: dimension 0 is d, the others are ordered by stride
     const int c1 = a.kdim_tok == 1 ? j0 : (a.kdim_head == 1 ? g : c.b);
     const int c2 = a.kdim_tok == 2 ? j0 : (a.kdim_head == 2 ? g : c.b);
     const int c3 = a.kdim_tok == 3 ? j0 : (a.kdim_head == 3 ? g : c.b);
-    tma_load_4d(dst, &a.kmap, 0, c1, c2, c3, fb, pol);
-    tma_load_4d(dst + kBoxBytes, &a.kmap, 64, c1, c2, c3, fb, pol);
+    if constexpr (F8) {
+      // 32 rows of 128 codes (one swizzled box) and the rows' 32 scales
+      mbar_arrive_expect_tx(fb, (uint32_t)(kSlotBytes + kT * 4));
+      tma_load_4d(dst, &a.kmap, 0, c1, c2, c3, fb, pol);
+      bulk_g2s(scale0 + s * kT * 4, a.kscale + ((int64_t)c.b * Hkv + g) * a.cap32 + j0, kT * 4, fb, pol);
+    } else {
+      mbar_arrive_expect_tx(fb, (uint32_t)kKBytes);
+      tma_load_4d(dst, &a.kmap, 0, c1, c2, c3, fb, pol);
+      tma_load_4d(dst + kBoxBytes, &a.kmap, 64, c1, c2, c3, fb, pol);
+    }
   };
 
   // prologue: the first kSW stages of this warp
@@ -183,17 +193,52 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
 
   // q of this warp's heads for the current sequence, as mma B fragments:
   // column grp is query head g*G + grp (zero for grp >= G), k = 16*kb + 2*tig (+8)
-  uint32_t bq[kMaxNg][8][2];
+  // F8: the same rows cast to E4M3 with one scale per head, as m16n8k32 B
+  // fragments (k = 32*kb + 4*tig .. +3, and +16), and the scales of this
+  // lane's accumulator columns (heads 2*tig and 2*tig + 1)
+  uint32_t bq[kMaxNg][F8 ? 4 : 8][2];
+  float sqA[kMaxNg], sqB[kMaxNg];
   auto load_q = [&](int b) {
-    const auto* q32 = static_cast<const uint32_t*>(a.q);
 #pragma unroll
     for (int r = 0; r < kMaxNg; ++r) {
       const bool has = r < ng && grp < G;
-      const int64_t row = has ? ((int64_t)b * a.q_sb + (int64_t)((warp + r * kNW) * G + grp) * a.q_sh) / 2 : 0;
+      const int64_t row = has ? (int64_t)b * a.q_sb + (int64_t)((warp + r * kNW) * G + grp) * a.q_sh : 0;
+      if constexpr (F8) {
+        const auto* qh = static_cast<const uint16_t*>(a.q) + row;
+        float v[4][8];
+        float amax = 0.f;
 #pragma unroll
-      for (int kb = 0; kb < 8; ++kb) {
-        bq[r][kb][0] = has ? __ldg(q32 + row + kb * 8 + tig) : 0u;
-        bq[r][kb][1] = has ? __ldg(q32 + row + kb * 8 + 4 + tig) : 0u;
+        for (int kb = 0; kb < 4; ++kb) {
+          uint2 lo{0u, 0u}, hi{0u, 0u};
+          if (has) {
+            lo = __ldg(reinterpret_cast<const uint2*>(qh + kb * 32 + 4 * tig));
+            hi = __ldg(reinterpret_cast<const uint2*>(qh + kb * 32 + 16 + 4 * tig));
+          }
+          to_float8<DT>(uint4{lo.x, lo.y, hi.x, hi.y}, v[kb]);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) amax = fmaxf(amax, fabsf(v[kb][i]));
+        }
+        amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 1));
+        amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 2));   // the head's 4 lanes hold all 128 dims
+        const float rq = amax > 0.f ? __fdiv_rn(448.f, amax) : 0.f;
+#pragma unroll
+        for (int kb = 0; kb < 4; ++kb) {
+          bq[r][kb][0] = e4m3x2(__fmul_rn(v[kb][0], rq), __fmul_rn(v[kb][1], rq)) |
+                         (e4m3x2(__fmul_rn(v[kb][2], rq), __fmul_rn(v[kb][3], rq)) << 16);
+          bq[r][kb][1] = e4m3x2(__fmul_rn(v[kb][4], rq), __fmul_rn(v[kb][5], rq)) |
+                         (e4m3x2(__fmul_rn(v[kb][6], rq), __fmul_rn(v[kb][7], rq)) << 16);
+        }
+        const float sq = amax > 0.f ? __fdiv_rn(amax, 448.f) : 0.f;
+        sqA[r] = __shfl_sync(0xffffffffu, sq, 8 * tig);
+        sqB[r] = __shfl_sync(0xffffffffu, sq, 8 * tig + 4);
+      } else {
+        const auto* q32 = static_cast<const uint32_t*>(a.q);
+#pragma unroll
+        for (int kb = 0; kb < 8; ++kb) {
+          bq[r][kb][0] = has ? __ldg(q32 + row / 2 + kb * 8 + tig) : 0u;
+          bq[r][kb][1] = has ? __ldg(q32 + row / 2 + kb * 8 + 4 + tig) : 0u;
+        }
+        sqA[r] = sqB[r] = 1.f;
       }
     }
   };
@@ -258,17 +303,28 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
         break;
       }
       const uint32_t sb = stage0 + cs * kSlotBytes;
-      // K tile -> A fragments (2 blocks of 16 tokens x 8 blocks of 16 dims)
-      uint32_t af[2][8][4];
+      // K tile -> A fragments: 16-bit keys, 2 blocks of 16 tokens x 8 blocks
+      // of 16 dims; E4M3 codes, 2 blocks of 16 tokens x 4 blocks of 32 dims
+      constexpr int kKB = F8 ? 4 : 8;
+      uint32_t af[2][kKB][4];
 #pragma unroll
       for (int mb = 0; mb < 2; ++mb) {
         const int t = mb * 16 + lm_row;
 #pragma unroll
-        for (int kb = 0; kb < 8; ++kb) {
-          const int chunk = kb * 2 + lm_khalf;          // 16-byte chunk of the 256-byte row
-          const uint32_t addr = sb + (chunk >> 3) * kBoxBytes + t * 128 + (((chunk & 7) ^ (t & 7)) << 4);
+        for (int kb = 0; kb < kKB; ++kb) {
+          const int chunk = kb * 2 + lm_khalf;   // 16-byte chunk of the row
+          const uint32_t addr = F8 ? sb + t * 128 + ((chunk ^ (t & 7)) << 4)
+                                   : sb + (chunk >> 3) * kBoxBytes + t * 128 + (((chunk & 7) ^ (t & 7)) << 4);
           ldmatrix_x4(addr, af[mb][kb]);
         }
+      }
+      // F8: the scales of this lane's token rows mb*16 + grp (+8)
+      float ksc[4] = {1.f, 1.f, 1.f, 1.f};
+      if constexpr (F8) {
+        const uint32_t sc = scale0 + cs * kT * 4;
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          ksc[u] = __uint_as_float(lds32(sc + ((u >> 1) * 16 + grp + (u & 1) * 8) * 4));
       }
       ++used;
       cph ^= (cs + 1 == (uint32_t)kSW) ? 1u : 0u;
@@ -290,9 +346,19 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
 #pragma unroll
         for (int e = 0; e < 4; ++e) acc[mb][e] = 0.f;
 #pragma unroll
-      for (int kb = 0; kb < 8; ++kb)
+      for (int kb = 0; kb < kKB; ++kb)
 #pragma unroll
-        for (int mb = 0; mb < 2; ++mb) mma_16816<DT>(acc[mb], af[mb][kb], bq[r][kb][0], bq[r][kb][1]);
+        for (int mb = 0; mb < 2; ++mb) {
+          if constexpr (F8) mma_16832_e4m3(acc[mb], af[mb][kb], bq[r][kb][0], bq[r][kb][1]);
+          else mma_16816<DT>(acc[mb], af[mb][kb], bq[r][kb][0], bq[r][kb][1]);
+        }
+      if constexpr (F8) {   // back to the key and query scales
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          acc[u >> 1][(u & 1) * 2] *= sqA[r] * ksc[u];
+          acc[u >> 1][(u & 1) * 2 + 1] *= sqB[r] * ksc[u];
+        }
+      }
 
       // acc[mb][c] = token mb*16 + grp, column 2*tig + c; acc[mb][2 + c] = token
       // mb*16 + grp + 8.  Columns >= G are zero (their q fragments are zero).
@@ -462,40 +528,40 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   }
 }
 
-template <int DT, int G, bool RAW>
+template <int DT, int G, bool RAW, bool F8>
 cudaError_t launch_score_t(const ScoreArgs& a, int grid, cudaStream_t st) {
-  const size_t smem = score_smem_bytes(G);
-  auto kern = hill_score_kernel<DT, G, RAW>;
+  const size_t smem = (size_t)ScoreCfg<G, F8>::kBytes;
+  auto kern = hill_score_kernel<DT, G, RAW, F8>;
   static int cache[64] = {0};
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), (int)smem, cache);
   if (e != cudaSuccess) return e;
   return launch_pdl(kern, dim3(grid), dim3(kThreads), smem, st, 0, a);
 }
 
-template <int DT, bool RAW>
+template <int DT, bool RAW, bool F8>
 cudaError_t launch_score_g(const ScoreArgs& a, int G, int grid, cudaStream_t st) {
   switch (G) {
-    case 1: return launch_score_t<DT, 1, RAW>(a, grid, st);
-    case 2: return launch_score_t<DT, 2, RAW>(a, grid, st);
-    case 4: return launch_score_t<DT, 4, RAW>(a, grid, st);
-    case 8: return launch_score_t<DT, 8, RAW>(a, grid, st);
+    case 1: return launch_score_t<DT, 1, RAW, F8>(a, grid, st);
+    case 2: return launch_score_t<DT, 2, RAW, F8>(a, grid, st);
+    case 4: return launch_score_t<DT, 4, RAW, F8>(a, grid, st);
+    case 8: return launch_score_t<DT, 8, RAW, F8>(a, grid, st);
   }
   return cudaErrorInvalidValue;
 }
 
-template <int G>
-size_t smem_for() {
-  return (size_t)ScoreCfg<G>::kBytes;
+template <int DT, bool F8>
+cudaError_t launch_score_m(const ScoreArgs& a, int G, bool raw, int grid, cudaStream_t st) {
+  return raw ? launch_score_g<DT, true, F8>(a, G, grid, st) : launch_score_g<DT, false, F8>(a, G, grid, st);
 }
 
 }  // namespace
 
-size_t score_smem_bytes(int G) {
+size_t score_smem_bytes(int G, bool f8) {
   switch (G) {
-    case 1: return smem_for<1>();
-    case 2: return smem_for<2>();
-    case 4: return smem_for<4>();
-    default: return smem_for<8>();
+    case 1: return f8 ? ScoreCfg<1, true>::kBytes : ScoreCfg<1, false>::kBytes;
+    case 2: return f8 ? ScoreCfg<2, true>::kBytes : ScoreCfg<2, false>::kBytes;
+    case 4: return f8 ? ScoreCfg<4, true>::kBytes : ScoreCfg<4, false>::kBytes;
+    default: return f8 ? ScoreCfg<8, true>::kBytes : ScoreCfg<8, false>::kBytes;
   }
 }
 
@@ -507,9 +573,9 @@ int score_max_kv_heads(int G) {
   return kMaxNg * kNW;
 }
 
-cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, int grid, cudaStream_t st) {
-  if (dtype == 0) return raw ? launch_score_g<0, true>(a, G, grid, st) : launch_score_g<0, false>(a, G, grid, st);
-  return raw ? launch_score_g<1, true>(a, G, grid, st) : launch_score_g<1, false>(a, G, grid, st);
+cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8, int grid, cudaStream_t st) {
+  if (dtype == 0) return f8 ? launch_score_m<0, true>(a, G, raw, grid, st) : launch_score_m<0, false>(a, G, raw, grid, st);
+  return f8 ? launch_score_m<1, true>(a, G, raw, grid, st) : launch_score_m<1, false>(a, G, raw, grid, st);
 }
 
 cudaError_t launch_attn_finalize(const FinalizeArgs& a, cudaStream_t st) {

@@ -8,7 +8,7 @@ fails loudly if the library has not been built.
 
 Names follow the C ABI: :func:`hill_score`, :func:`hill_topk_select`,
 :func:`hill_gather_sparse_attn`, :func:`hill_evict_step`, :func:`hill_topk_select_bkp`,
-:func:`hill_evict_step_bkp`,
+:func:`hill_evict_step_bkp`, :func:`hill_quantize_k`, :func:`hill_score_f8`, :func:`hill_evict_step_f8`,
 :func:`hill_workspace_bytes`, :func:`hill_sync_status`.
 """
 from __future__ import annotations
@@ -73,6 +73,9 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_evict_step.argtypes = [D, P, P, P, P, P, I32, I32, P, P, P, P, P, P, SZ, P]
     lib.hill_topk_select_bkp.argtypes = [D, P, P, P, I32, I32, P, P, P, P, SZ, P]
     lib.hill_evict_step_bkp.argtypes = [D, P, P, P, P, P, I32, I32, I32, P, P, P, P, P, P, P, SZ, P]
+    lib.hill_quantize_k.argtypes = [D, P, P, P, I32, P, P, P]
+    lib.hill_score_f8.argtypes = [D, P, P, P, P, I32, P, P, P, SZ, P]
+    lib.hill_evict_step_f8.argtypes = [D, P, P, P, P, P, P, P, I32, I32, P, P, P, P, P, P, SZ, P]
     lib.hill_score_noalloc.argtypes = [D, P, P, P, I32, P, P, P]
     lib.hill_score_noalloc.restype = I32
     lib.hill_sync_status.argtypes = [P]
@@ -81,7 +84,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_abi_version.restype = I32
     lib.hill_kernel_launches.restype = ctypes.c_uint64
     for name in ("hill_score", "hill_topk_select", "hill_gather_sparse_attn", "hill_evict_step",
-                 "hill_topk_select_bkp", "hill_evict_step_bkp", "hill_sync_status"):
+                 "hill_topk_select_bkp", "hill_evict_step_bkp", "hill_quantize_k", "hill_score_f8",
+                 "hill_evict_step_f8", "hill_sync_status"):
         getattr(lib, name).restype = I32
     _lib = lib
     return lib
@@ -202,6 +206,38 @@ def hill_evict_step_bkp(desc, q, k_cache, v_cache, lens, k, recent, max_k, mode,
                                       _ptr(k), int(recent), int(max_k), int(mode), _ptr(accum), _ptr(scores),
                                       _ptr(idx), _ptr(count), _ptr(hits), _ptr(out), wp, wn,
                                       _stream(stream)), "hill_evict_step_bkp")
+
+
+def shadow_shape(desc):
+    """Shapes of the E4M3 key shadow: (codes [B][Hkv][cap][128], scales [B][Hkv][cap32])."""
+    cap32 = (desc.capacity + 31) // 32 * 32
+    return ((desc.batch, desc.num_kv_heads, desc.capacity, desc.head_dim),
+            (desc.batch, desc.num_kv_heads, cap32))
+
+
+def alloc_shadow(desc, device="cuda"):
+    cs, ss = shadow_shape(desc)
+    return torch.zeros(cs, dtype=torch.uint8, device=device), torch.zeros(ss, dtype=torch.float32, device=device)
+
+
+def hill_quantize_k(desc, k_cache, row_begin, row_end, max_rows, k8, kscale, stream=None) -> None:
+    _check(load().hill_quantize_k(ctypes.byref(desc), _ptr(k_cache), _ptr(row_begin), _ptr(row_end),
+                                  int(max_rows), _ptr(k8), _ptr(kscale), _stream(stream)), "hill_quantize_k")
+
+
+def hill_score_f8(desc, q, k8, kscale, lens, mode, scores, accum=None, ws=None, stream=None) -> None:
+    wp, wn = _ws(ws)
+    _check(load().hill_score_f8(ctypes.byref(desc), _ptr(q), _ptr(k8), _ptr(kscale), _ptr(lens), int(mode),
+                                _ptr(scores), _ptr(accum), wp, wn, _stream(stream)), "hill_score_f8")
+
+
+def hill_evict_step_f8(desc, q, k8, kscale, k_cache, v_cache, lens, k, max_k, mode, accum, scores, idx, count,
+                       out, ws, stream=None) -> None:
+    wp, wn = _ws(ws)
+    _check(load().hill_evict_step_f8(ctypes.byref(desc), _ptr(q), _ptr(k8), _ptr(kscale), _ptr(k_cache),
+                                     _ptr(v_cache), _ptr(lens), _ptr(k), int(max_k), int(mode), _ptr(accum),
+                                     _ptr(scores), _ptr(idx), _ptr(count), _ptr(out), wp, wn, _stream(stream)),
+           "hill_evict_step_f8")
 
 
 def hill_kernel_launches() -> int:

@@ -23,13 +23,14 @@ def lib():
 def _declared():
     text = open(HEADER).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(hill_[a-z_]+)\s*\(", text)))
+    return sorted(set(re.findall(r"\b(hill_[a-z0-9_]+)\s*\(", text)))
 
 
 def test_header_declares_the_boundary():
     names = _declared()
     for n in ("hill_score", "hill_topk_select", "hill_gather_sparse_attn", "hill_evict_step",
-              "hill_topk_select_bkp", "hill_evict_step_bkp",
+              "hill_topk_select_bkp", "hill_evict_step_bkp", "hill_quantize_k", "hill_score_f8",
+              "hill_evict_step_f8",
               "hill_workspace_bytes", "hill_sync_status", "hill_status_string", "hill_abi_version"):
         assert n in names
 
@@ -96,6 +97,13 @@ def test_host_validation_without_device(lib):
     assert lib.hill_gather_sparse_attn(ctypes.byref(d), FAKE, FAKE, None, FAKE, FAKE, 8, FAKE, None, 0,
                                        None) == INV
     assert lib.hill_workspace_bytes(ctypes.byref(_desc(head_dim=64)), 0, 8) == 0
+    # E4M3 shadow: missing or misaligned shadow arrays are rejected before any device work
+    assert lib.hill_quantize_k(ctypes.byref(d), FAKE, FAKE, FAKE, 1, None, FAKE, None) == INV
+    assert lib.hill_quantize_k(ctypes.byref(d), FAKE, FAKE, FAKE, -1, FAKE, FAKE, None) == INV
+    assert lib.hill_score_f8(ctypes.byref(d), FAKE, FAKE + 8, FAKE, FAKE, 0, FAKE, None, FAKE, 1 << 30,
+                             None) == INV
+    assert lib.hill_evict_step_f8(ctypes.byref(d), FAKE, FAKE, None, None, None, FAKE, FAKE, 8, 0, None, None,
+                                  FAKE, FAKE, None, FAKE, 1 << 30, None) == INV
     # BKP: a negative window is rejected before any device work
     assert lib.hill_topk_select_bkp(ctypes.byref(d), FAKE, FAKE, FAKE, -1, 8, FAKE, FAKE, None, None, 0,
                                     None) == INV
