@@ -264,11 +264,28 @@ def run_ours(args):
     stream = torch.cuda.Stream(device=dev)
 
     hits = torch.zeros(lres, B, cap, dtype=torch.int16, device=dev) if bkp else None
+    f8 = args.f8
+    if f8:
+        # E4M3 shadow of every resident layer's keys (Sec. 4.4), built before
+        # timing; every decode step re-quantises its appended token row
+        cs, ss = hill.shadow_shape(desc)
+        k8_all = torch.zeros((lres,) + cs, dtype=torch.uint8, device=dev)
+        ks_all = torch.zeros((lres,) + ss, dtype=torch.float32, device=dev)
+        zeros_b = torch.zeros(B, dtype=torch.int32, device=dev)
+        cap_b = torch.full((B,), cap, dtype=torch.int32, device=dev)
+        for r in range(lres):
+            hill.hill_quantize_k(desc, Kall[r], zeros_b, cap_b, cap, k8_all[r], ks_all[r])
+        new_row = lens_all - 1
+        torch.cuda.synchronize()
 
     def evict(t, l, o, st):
         r = l % lres
         acc = accum[r] if accum is not None else None
-        if bkp:
+        if f8:
+            hill.hill_quantize_k(desc, Kall[r], new_row[t], lens_all[t], 1, k8_all[r], ks_all[r], st)
+            hill.hill_evict_step_f8(desc, q_all[t, l], k8_all[r], ks_all[r], Kall[r], Vall[r], lens_all[t], k_all[t],
+                                    max_k, mode, acc, scores[l], idx[l], count[l], o, ws, st)
+        elif bkp:
             hill.hill_evict_step_bkp(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], args.bkp_recent,
                                      max_k, mode, acc, scores[l], idx[l], count[l], hits[r], o, ws, st)
         else:
@@ -325,7 +342,9 @@ def run_ours(args):
     ms = max_over_ranks(ms_local, dev)
     tokens = sum(tokens_of[t] for t in order)
     value = world * tokens / (ms / 1e3)
-    k_bytes_per_token = Hkv * d * 2
+    # bytes of the key stream the scoring reads per token: the 16-bit keys, or
+    # with --f8 the E4M3 codes and one float32 scale per row
+    k_bytes_per_token = Hkv * (d + 4) if f8 else Hkv * d * 2
     k_gbs = world * tokens * k_bytes_per_token / (ms / 1e3) / 1e9
     gpu_launches = sum(launches[t] for t in order)
 
@@ -377,7 +396,11 @@ def run_ours(args):
                 r = l % lres
                 if rep == 1:
                     starts[l].record(stream)
-                hill.hill_score(desc, q_all[t_s, l], Kall[r], lens_all[t_s], mode, scores[l], None, ws, stream)
+                if f8:
+                    hill.hill_score_f8(desc, q_all[t_s, l], k8_all[r], ks_all[r], lens_all[t_s], mode, scores[l],
+                                       None, ws, stream)
+                else:
+                    hill.hill_score(desc, q_all[t_s, l], Kall[r], lens_all[t_s], mode, scores[l], None, ws, stream)
                 if rep == 1:
                     ends[l].record(stream)
     stream.synchronize()
@@ -393,9 +416,10 @@ def run_ours(args):
         else "hill_score: hill_score_kernel",
         "bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
         "frac": round(achieved / peak, 4), "peak_source": peak_kind,
-        "traffic": profile_traffic("hill_score_" + args.mode, w.name),
+        "traffic": profile_traffic("hill_score_" + args.mode + ("_f8" if f8 else ""), w.name),
         "algorithmic_bytes_per_launch": alg_bytes,
-        "bytes_per_token": f"Hkv*d*2 + 4 = {k_bytes_per_token + 4}",
+        "bytes_per_token": (f"Hkv*(d+4) + 4 = {k_bytes_per_token + 4}" if f8
+                            else f"Hkv*d*2 + 4 = {k_bytes_per_token + 4}"),
         "launch_us": round(score_ms * 1e3, 2),
     }
 
@@ -415,7 +439,8 @@ def run_ours(args):
             "warmup": args.warmup, "ms_per_step": round(ms / len(order), 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f16" if w.dtype == torch.float16 else "bf16",
             "data": "synthetic", "config": dict(describe(w, lres, args.mode),
-                                                **({"bkp_recent": args.bkp_recent} if bkp else {})),
+                                                **({"bkp_recent": args.bkp_recent} if bkp else {}),
+                                                **({"scoring": "e4m3 key shadow"} if f8 else {})),
             "k_stream_gbs": round(k_gbs, 1),
             "k_stream_frac_of_measured_hbm": round(k_gbs / world / peak, 4),
             "k_stream_frac_of_8tbs": round(k_gbs / world / 8000.0, 4),
@@ -586,6 +611,8 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--f8", action="store_true",
+                    help="asymmetric-precision scoring (Sec. 4.4) from an E4M3 key shadow (hill_evict_step_f8)")
     ap.add_argument("--bkp-recent", type=int, default=-1,
                     help="BKP bookkeeping (Sec. 4.2): pin this many recent tokens and keep a hit-rate table "
                          "(hill_evict_step_bkp); default off")

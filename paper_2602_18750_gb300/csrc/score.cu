@@ -2,8 +2,13 @@
 // the ATTN-mode normalisation (Sec. 4.1 column sum of softmax weights).
 //
 // hill_score_kernel: persistent CTAs of kNW warps.  A work item is a tile of
-// kT = 32 consecutive tokens of one sequence; the KV heads g of an item are
-// dealt to the warps (g mod kNW).  Every warp streams its own (item, g)
+// kT = 32 consecutive tokens of one sequence; CTA x takes the contiguous
+// range of items [x * per, (x + 1) * per), so it meets one or two sequences
+// and loads their queries and flushes their partials once (measured faster
+// than dealing items round robin, by 4 % at 32K and more for short
+// sequences, where round robin changes sequence at every item).  The KV
+// heads g of an item are dealt to the warps (g mod kNW).  Every warp streams
+// its own (item, g)
 // sequence through a private ring of kSW shared-memory stages: lane 0 issues
 // two tiled TMA loads (dims 0-63 and 64-127 of the tile's 32 key rows, 128-
 // byte swizzle) completing on the stage's mbarrier.  The warp moves a landed tile into
@@ -131,19 +136,21 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   }
   __syncthreads();
   const int n_items = tstart[B];
-  if ((int)blockIdx.x >= n_items) return;
+  const int per = (n_items + gridDim.x - 1) / gridDim.x;     // items per CTA
+  const int it_lo = min(n_items, (int)blockIdx.x * per), it_hi = min(n_items, it_lo + per);
+  if (it_lo >= it_hi) return;
   const int ng = (Hkv - warp + kNW - 1) / kNW;   // KV heads of this warp per tile (0 .. kMaxNg)
 
   const uint64_t pol = l2_evict_first_policy();
   const uint32_t stage0 = base_addr + warp * kSW * kSlotBytes;
   const uint32_t bar0 = base_addr + Cfg::kOffBar + warp * kSW * 8;
   const uint32_t scale0 = base_addr + Cfg::kOffScale + warp * kSW * kT * 4;   // F8 only
-  const int b_first = find_seq(tstart, B, blockIdx.x);
+  const int b_first = find_seq(tstart, B, it_lo);
 
   auto advance = [&](Cursor& c) {
     if (++c.r >= ng) {
       c.r = 0;
-      c.item += gridDim.x;
+      ++c.item;
       while (c.b < B - 1 && tstart[c.b + 1] <= c.item) ++c.b;
     }
   };
@@ -170,10 +177,10 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   };
 
   // prologue: the first kSW stages of this warp
-  Cursor pc{(int)blockIdx.x, 0, b_first};
+  Cursor pc{it_lo, 0, b_first};
   uint32_t issued = 0, is_slot = 0;
   if (ng > 0) {
-    for (; issued < (uint32_t)kSW && pc.item < n_items; ++issued) {
+    for (; issued < (uint32_t)kSW && pc.item < it_hi; ++issued) {
       if (lane == 0) issue(pc, is_slot);
       is_slot = is_slot + 1 == (uint32_t)kSW ? 0u : is_slot + 1;
       advance(pc);
@@ -278,7 +285,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
     }
   };
 
-  for (int item = blockIdx.x, b = b_first; item < n_items; item += gridDim.x, ++item_no) {
+  for (int item = it_lo, b = b_first; item < it_hi; ++item, ++item_no) {
     while (b < B - 1 && tstart[b + 1] <= item) ++b;
     const int tile = item - tstart[b];
     const int j0 = tile * kT;
@@ -290,7 +297,8 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
       load_q(b);
       if (!RAW) reset_stat();
       cur_b = b;
-      cur_slot = tile;   // = item - tstart[b]: this CTA's first item in b (< gridDim.x)
+      // this CTA's partial slot in b: its rank among the CTAs whose ranges meet b
+      cur_slot = (int)blockIdx.x - tstart[b] / per;
     }
 
 #pragma unroll
@@ -331,7 +339,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
       const uint32_t freed = cs;
       cs = cs + 1 == (uint32_t)kSW ? 0u : cs + 1;
       __syncwarp();
-      if (pc.item < n_items) {   // the slot just read takes the stage kSW ahead
+      if (pc.item < it_hi) {   // the slot just read takes the stage kSW ahead
         if (lane == 0) {
           fence_proxy_async_smem();
           issue(pc, freed);
@@ -458,8 +466,28 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   float zr[kFinZReg];
 #pragma unroll
   for (int u = 0; u < kFinZReg; ++u) zr[u] = (valid && u < a.H) ? zp[(int64_t)u * a.cap] : 0.f;
+  // the scoring CTAs that met b wrote slots 0 .. ns-1
+  // (every thread counts the tiles of a share of the sequences)
+  __shared__ int s_first, s_total;
+  if (threadIdx.x == 0) s_first = s_total = 0;
+  __syncthreads();
+  {
+    int f = 0, t = 0;
+    for (int bb = threadIdx.x; bb < a.B; bb += kFinThreads) {
+      int lb = a.lens[bb];
+      lb = lb < 0 ? 0 : (lb > a.cap ? a.cap : lb);
+      const int tiles = (lb + kT - 1) / kT;
+      f += bb < b ? tiles : 0;
+      t += tiles;
+    }
+    if (f) atomicAdd(&s_first, f);
+    if (t) atomicAdd(&s_total, t);
+  }
+  __syncthreads();
+  const int first_item = s_first;
+  const int per = (s_total + a.nslot - 1) / a.nslot;
   const int items = (len + kT - 1) / kT;
-  const int ns = min(items, a.nslot);
+  const int ns = (first_item + items - 1) / per - first_item / per + 1;
   const float2* pb = a.partials + (int64_t)b * a.nslot * a.H;
   const int sub = threadIdx.x % kFinPartThreads;
   for (int h = threadIdx.x / kFinPartThreads; h < a.H; h += kFinThreads / kFinPartThreads) {
