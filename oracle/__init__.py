@@ -19,6 +19,8 @@ arrays into it.  Each wrapper names the part of the paper it follows:
 * :func:`bkp_select`   -- BKP pinning + hit-rate table (Sec. 4.2)
 * :func:`sparse_attn`  -- attention over the selected KV only (Sec. 4.1, workflow step 6)
 * :func:`evict_step`   -- the five steps in order
+* :func:`scores_kvh`, :func:`topk_kvh`, :func:`sparse_attn_kvh` -- the per-KV-head
+                          selection variant, composed from the functions above
 
 Pins: tests/test_oracle_pins.py checks every function against library
 routines (torch fp64 matmul / softmax / topk / scaled_dot_product_attention),
@@ -248,6 +250,39 @@ def bkp_select(key, lens, k, recent, max_k, hits=None):
     rc = _load().oracle_bkp_select(B, cap, _ptr(_i32(lens)), _ptr(key), _ptr(_i32(k)), int(recent),
                                    max_k, _ptr(idx), _ptr(count), _ptr(h))
     return idx, count, rc, h
+
+
+def scores_kvh(mode, z, lens, Hkv) -> np.ndarray:
+    """Per-KV-head importance s[B][Hkv][cap]: Step 2 restricted to the G query
+    heads of each KV head (the same softmax per (b, h), summed within the
+    group only), i.e. :func:`scores` on z regrouped as [B*Hkv][G][cap]."""
+    z = np.ascontiguousarray(z, dtype=np.float64)
+    B, H, cap = z.shape
+    G = H // Hkv
+    s = scores(mode, z.reshape(B * Hkv, G, cap), np.repeat(_i32(lens), Hkv))
+    return s.reshape(B, Hkv, cap)
+
+
+def topk_kvh(key, lens, k, max_k):
+    """One top-k per (b, g) row of key[B][Hkv][cap] (budget k[b] for every g):
+    (idx[B][Hkv][max_k], count[B][Hkv], rc)."""
+    key = np.ascontiguousarray(key, dtype=np.float64)
+    B, Hkv, cap = key.shape
+    idx, count, rc = topk(key.reshape(B * Hkv, cap), np.repeat(_i32(lens), Hkv), np.repeat(_i32(k), Hkv), max_k)
+    return idx.reshape(B, Hkv, max_k), count.reshape(B, Hkv), rc
+
+
+def sparse_attn_kvh(q, K, V, idx, count, dtype=None) -> np.ndarray:
+    """Attention where the query heads of KV head g read only the rows
+    idx[b][g][:count[b][g]]: :func:`sparse_attn` per KV head."""
+    Hkv = K.shape[1]
+    H = q.shape[1]
+    G = H // Hkv
+    idx = np.asarray(idx)
+    count = np.asarray(count)
+    outs = [sparse_attn(q[:, g * G:(g + 1) * G], K[:, g:g + 1], V[:, g:g + 1], idx[:, g], count[:, g], dtype)
+            for g in range(Hkv)]
+    return np.concatenate(outs, axis=1)
 
 
 def sparse_attn(q, K, V, idx, count, dtype=None) -> np.ndarray:

@@ -311,6 +311,56 @@ def test_logits_q8_lossless_rows_equal_exact_logits(oracle_mod):
     assert np.allclose(z8, z, rtol=1e-12, atol=0)
 
 
+# ---------------------------------------------------------------- per-KV-head selection
+def test_kvh_reduces_to_sequence_path_for_one_kv_head(oracle_mod):
+    """With Hkv = 1 the per-KV-head scores, selection and attention are the
+    per-sequence ones."""
+    B, H, d, cap = 2, 4, 64, 50
+    lens, k = [50, 31], [9, 31]
+    q, K, V, _ = inputs.random_case(B, H, 1, d, cap, lens, seed=14)
+    z = oracle_mod.logits(q, K, lens)
+    for mode in (oracle_mod.ATTN, oracle_mod.RAW):
+        s1 = oracle_mod.scores_kvh(mode, z, lens, 1)
+        s0 = oracle_mod.scores(mode, z, lens)
+        assert np.allclose(s1[:, 0], s0, equal_nan=True, rtol=0, atol=0)
+        i1, c1, _ = oracle_mod.topk_kvh(s1, lens, k, 32)
+        i0, c0, _ = oracle_mod.topk(s0, lens, k, 32)
+        assert np.array_equal(i1[:, 0], i0) and np.array_equal(c1[:, 0], c0)
+        o1 = oracle_mod.sparse_attn_kvh(q, K, V, i1, c1)
+        o0 = oracle_mod.sparse_attn(q, K, V, i0, c0)
+        assert np.array_equal(o1, o0)
+
+
+def test_kvh_mha_selects_each_heads_own_softmax_top(oracle_mod):
+    """MHA (G = 1), ATTN: each KV head keeps the top-k of its own softmax row,
+    which is the top-k of its logits (softmax is monotone) -- checked against
+    torch.topk on the logits; the per-head mass is 1 (Σ_j p = 1)."""
+    B, H, d, cap = 1, 6, 64, 40
+    lens, k = [40], [7]
+    q, K, V, _ = inputs.random_case(B, H, H, d, cap, lens, seed=15)
+    z = oracle_mod.logits(q, K, lens)
+    s = oracle_mod.scores_kvh(oracle_mod.ATTN, z, lens, H)
+    assert np.allclose(s[0].sum(axis=1), 1.0)
+    idx, cnt, _ = oracle_mod.topk_kvh(s, lens, k, 7)
+    for g in range(H):
+        want = sorted(torch.topk(torch.from_numpy(z[0, g]), 7).indices.tolist())
+        assert idx[0, g].tolist() == want
+
+
+def test_kvh_attention_uses_each_heads_rows(oracle_mod):
+    """GQA: query heads of KV head g attend over idx[b][g] only -- a one-token
+    set gives that token's V row of head g for all G query heads."""
+    B, H, Hkv, d, cap = 1, 4, 2, 32, 12
+    q, K, V, _ = inputs.random_case(B, H, Hkv, d, cap, [12], seed=16)
+    idx = np.array([[[3, 0], [10, 0]]], dtype=np.int32)
+    cnt = np.array([[1, 1]], dtype=np.int32)
+    o = oracle_mod.sparse_attn_kvh(q, K, V, idx, cnt)
+    Vd = oracle_mod.decode16(V)
+    for h in range(H):
+        g = h // 2
+        assert np.allclose(o[0, h], Vd[0, g, idx[0, g, 0]])
+
+
 # ---------------------------------------------------------------- BKP bookkeeping (Sec. 4.2)
 def test_bkp_without_window_is_topk(oracle_mod):
     """recent = 0 reduces BKP selection to the pinned top-k, and the hit table
