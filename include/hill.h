@@ -153,6 +153,22 @@ hill_status hill_evict_step_bkp(const hill_desc* desc, const void* q, const void
                                 float* scores, int32_t* idx, int32_t* count, uint16_t* hits, float* out,
                                 void* ws, size_t ws_bytes, void* stream);
 
+/* Per-KV-head selection (a variant of the evaluation: the paper evaluates at
+ * token level for every head topology, Sec. 5.3; here each KV head keeps its
+ * own set).  The importance is aggregated over the G query heads of each KV
+ * head only,
+ *   ATTN: s[b][g][j] = sum_{h in group g} softmax_{j'<lens[b]}(z[b,h,j'])[j]
+ *   RAW : s[b][g][j] = sum_{h in group g} z[b,h,j],
+ * written to scores [B][Hkv][cap] (caller-owned, required unless accum
+ * [B][Hkv][cap] is given; then accum += s and the ranking uses accum).  The
+ * top min(k[b], lens[b]) tokens of every (b, g) go to idx [B][Hkv][max_k]
+ * (ascending, -1 padded) and count [B][Hkv], and if out != NULL the query
+ * heads of KV head g attend over idx[b][g] only.  B * Hkv <= 512. */
+hill_status hill_evict_step_kvh(const hill_desc* desc, const void* q, const void* k_cache,
+                                const void* v_cache, const int32_t* lens, const int32_t* k, int32_t max_k,
+                                hill_score_mode mode, float* accum, float* scores, int32_t* idx,
+                                int32_t* count, float* out, void* ws, size_t ws_bytes, void* stream);
+
 /* Asymmetric-precision scoring (Sec. 4.4, CEC): the evaluation ranks tokens
  * with low-precision inner products, while the attention keeps the original
  * 16-bit keys and values.  On this GPU the low precision is OCP FP8 E4M3

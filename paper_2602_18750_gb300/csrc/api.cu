@@ -205,7 +205,7 @@ hill_status from_cuda(cudaError_t e) { return e == cudaSuccess ? HILL_OK : HILL_
 hill_status run_score(const hill_desc* d, const void* q, const void* k, const int32_t* lens, int mode,
                       float* scores, float* accum, unsigned char* base, const Layout& L,
                       const DeviceInfo& di, cudaStream_t st, uint32_t* hist0 = nullptr, int recent = 0,
-                      const float* kscale = nullptr) {
+                      const float* kscale = nullptr, bool kvh = false) {
   if (d->batch == 0 || d->capacity == 0) return HILL_OK;
   const int G = d->num_q_heads / d->num_kv_heads;
   ScoreArgs a{};
@@ -230,6 +230,7 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   a.kscale = kscale;
   a.cap32 = cap32_of(d);
   const bool raw = mode == HILL_SCORE_RAW;
+  a.kvh = kvh ? 1 : 0;
   if (raw) {
     a.scores = scores;
     a.accum = accum;
@@ -253,12 +254,15 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   f.accum = accum;
   f.hist0 = hist0;
   f.recent = recent;
+  f.kvh = kvh ? 1 : 0;
+  f.Hkv = d->num_kv_heads;
   return from_cuda(counted(launch_attn_finalize(f, st), 1));
 }
 
 hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens, const int32_t* k,
                        int max_k, int32_t* idx, int32_t* count, const DeviceInfo& di, cudaStream_t st,
-                       const uint32_t* hist0 = nullptr, int recent = 0, uint16_t* hits = nullptr) {
+                       const uint32_t* hist0 = nullptr, int recent = 0, uint16_t* hits = nullptr,
+                       bool kvh = false) {
   if (d->batch == 0) return HILL_OK;
   SelectArgs a{};
   a.key = key;
@@ -272,13 +276,15 @@ hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens
   a.hist0 = hist0;
   a.recent = recent;
   a.hits = hits;
+  a.rows_per_seq = kvh ? d->num_kv_heads : 1;
   a.err = di.err;
   return from_cuda(counted(launch_select(a, st), 1));
 }
 
 hill_status run_attn(const hill_desc* d, const void* q, const void* k, const void* v, const int32_t* idx,
                      const int32_t* count, int max_k, float* out, unsigned char* base, const Layout& L,
-                     const DeviceInfo& di, cudaStream_t st) {
+                     const DeviceInfo& di, cudaStream_t st,
+                     bool kvh = false) {
   if (d->batch == 0) return HILL_OK;
   // the gather forms row offsets as 32-bit stride x 32-bit index products
   if (d->k_sn > INT32_MAX || d->v_sn > INT32_MAX) return HILL_ERR_UNSUPPORTED;
@@ -304,6 +310,7 @@ hill_status run_attn(const hill_desc* d, const void* q, const void* k, const voi
   a.out = out;
   a.part = reinterpret_cast<float*>(base + L.attn_part);
   a.splits = L.splits;
+  a.kvh = kvh ? 1 : 0;
   a.err = di.err;
   return from_cuda(counted(launch_sparse_attn(a, d->dtype, d->num_q_heads / d->num_kv_heads, L.attn_grid, st), 2));
 }
@@ -446,6 +453,32 @@ hill_status hill_topk_select_bkp(const hill_desc* desc, const float* scores, con
   if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
   return run_select(desc, scores, lens, k, max_k, idx, count, di, static_cast<cudaStream_t>(stream), nullptr,
                     recent, hits);
+}
+
+hill_status hill_evict_step_kvh(const hill_desc* desc, const void* q, const void* k_cache, const void* v_cache,
+                                const int32_t* lens, const int32_t* k, int32_t max_k, hill_score_mode mode,
+                                float* accum, float* scores, int32_t* idx, int32_t* count, float* out, void* ws,
+                                size_t ws_bytes, void* stream) {
+  hill_status s = check_desc(desc);
+  if (s != HILL_OK) return s;
+  if (mode != HILL_SCORE_ATTN && mode != HILL_SCORE_RAW) return HILL_ERR_INVALID_ARG;
+  if (max_k < 0 || !q || !k_cache || !lens || !k || !count || (max_k > 0 && !idx) || (!scores && !accum))
+    return HILL_ERR_INVALID_ARG;
+  if (out && !v_cache) return HILL_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k_cache) || (out && !aligned16(v_cache))) return HILL_ERR_INVALID_ARG;
+  // the attention keeps one table entry per (b, g) on chip
+  if ((int64_t)desc->batch * desc->num_kv_heads > attn_max_batch()) return HILL_ERR_UNSUPPORTED;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  const Layout L = layout_for(desc, mode, max_k, di.sms);
+  if (!ws || ws_bytes < L.total) return HILL_ERR_WORKSPACE;
+  unsigned char* base = ws_base(ws);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  s = run_score(desc, q, k_cache, lens, mode, scores, accum, base, L, di, st, nullptr, 0, nullptr, true);
+  if (s != HILL_OK) return s;
+  s = run_select(desc, accum ? accum : scores, lens, k, max_k, idx, count, di, st, nullptr, 0, nullptr, true);
+  if (s != HILL_OK || !out) return s;
+  return run_attn(desc, q, k_cache, v_cache, idx, count, max_k, out, base, L, di, st, true);
 }
 
 hill_status hill_quantize_k(const hill_desc* desc, const void* k_cache, const int32_t* row_begin,

@@ -45,13 +45,15 @@ struct AttnCfg {
   static constexpr int kSmem = kAW * kNS * kSlotBytes + 128;   // + alignment slack
 };
 
-// Position of a batch in the list: sequence, KV head, batch within (b, g).
+// Position of a batch in the list: table unit u (a sequence b, or with
+// per-KV-head selection a pair (b, g)), sequence, KV head, batch within (b, g).
 struct Pos {
-  int b, g, bi;
+  int u, b, g, bi;
 };
 
-__device__ __forceinline__ int clamp_count(const AttnArgs& a, int b) {
-  const int n = a.count[b];
+// Selected-token count of table unit u (count[] has one entry per unit).
+__device__ __forceinline__ int clamp_count(const AttnArgs& a, int u) {
+  const int n = a.count[u];
   return n < 0 ? 0 : (n > a.max_k ? a.max_k : n);
 }
 
@@ -73,22 +75,27 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   pdl_wait();
   pdl_launch_dependents();
 
-  for (int b = threadIdx.x; b < a.B; b += kAThreads) {
-    const int n = clamp_count(a, b);
-    s_cnt[b] = n;
-    s_nbat[b] = (n + kBatch - 1) / kBatch;
+  // table units: sequences (every KV head reads the same set, Hkv * nbat
+  // batches per unit, ordered g, bi), or with per-KV-head selection the pairs
+  // (b, g) (nbat batches per unit)
+  const int R = a.kvh ? a.B * a.Hkv : a.B;
+  const int upb = a.kvh ? 1 : a.Hkv;   // KV heads per unit
+  for (int u = threadIdx.x; u < R; u += kAThreads) {
+    const int n = clamp_count(a, u);
+    s_cnt[u] = n;
+    s_nbat[u] = (n + kBatch - 1) / kBatch;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
     int acc = 0;
-    for (int b = 0; b < a.B; ++b) {
-      s_bstart[b] = acc;
-      acc += a.Hkv * s_nbat[b];
+    for (int u = 0; u < R; ++u) {
+      s_bstart[u] = acc;
+      acc += upb * s_nbat[u];
     }
-    s_bstart[a.B] = acc;
+    s_bstart[R] = acc;
   }
   __syncthreads();
-  const int total = s_bstart[a.B];
+  const int total = s_bstart[R];
   const int nwarps = gridDim.x * kAW;
   const int gw = blockIdx.x * kAW + warp;
   int t0, t1;
@@ -105,27 +112,33 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   // position of batch t0 (binary search once), then advanced one batch at a time
   Pos first;
   {
-    int lo = 0, hi = a.B;
+    int lo = 0, hi = R;
     while (hi - lo > 1) {
       const int mid = (lo + hi) >> 1;
       if (s_bstart[mid] <= t0) lo = mid; else hi = mid;
     }
     const int rem = t0 - s_bstart[lo];
-    first.b = lo;
-    first.g = rem / s_nbat[lo];
-    first.bi = rem - first.g * s_nbat[lo];
+    first.u = lo;
+    if (a.kvh) {
+      first.b = lo / a.Hkv;
+      first.g = lo - first.b * a.Hkv;
+      first.bi = rem;
+    } else {
+      first.b = lo;
+      first.g = rem / s_nbat[lo];
+      first.bi = rem - first.g * s_nbat[lo];
+    }
   }
   auto advance = [&](Pos& p) {
-    if (p.b >= a.B) return;
-    if (++p.bi >= s_nbat[p.b]) {
-      p.bi = 0;
-      if (++p.g >= a.Hkv) {
-        p.g = 0;
-        do {
-          ++p.b;
-        } while (p.b < a.B && s_nbat[p.b] == 0);
-      }
-    }
+    if (p.u >= R) return;
+    if (++p.bi < s_nbat[p.u]) return;
+    p.bi = 0;
+    if (!a.kvh && ++p.g < a.Hkv) return;
+    do {
+      ++p.u;
+    } while (p.u < R && s_nbat[p.u] == 0);
+    p.b = a.kvh ? p.u / a.Hkv : p.u;
+    p.g = a.kvh ? p.u - p.b * a.Hkv : 0;
   };
 
   // raw index entry of this lane for the batch at p (-1 past the count).
@@ -133,7 +146,7 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   // until the batch is issued one iteration later, where it is checked.
   auto load_idx = [&](const Pos& p) -> int {
     const int e = p.bi * kBatch + lane;
-    return e < s_cnt[p.b] ? a.idx[(int64_t)p.b * a.max_k + e] : -1;
+    return e < s_cnt[p.u] ? a.idx[(int64_t)p.u * a.max_k + e] : -1;
   };
   // gather the batch at p into slot s: row r of the batch is token jj of
   // lane r (-1: none, zero-filled).  A half-warp copies one 256-byte row;
@@ -143,7 +156,7 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   const uint32_t dst_lane = (uint32_t)((l16 >> 3) * kHalfBytes + hrow * 128);
   const uint32_t swz_lane = (uint32_t)(((l16 & 7) ^ hrow) << 4);
   auto issue = [&](const Pos& p, int s, int jj) -> unsigned {
-    if (p.bi * kBatch + lane < s_cnt[p.b] && (jj < 0 || jj >= a.cap)) {
+    if (p.bi * kBatch + lane < s_cnt[p.u] && (jj < 0 || jj >= a.cap)) {
       raise_error(a.err, kErrDevArg);   // a listed entry outside [0, cap): skipped
       jj = -1;
     }
@@ -197,7 +210,7 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   float m_run = -INFINITY, l_run = 0.f;       // softmax state of head grp (base 2)
   float oacc[8][4];
   uint32_t qa[8][2];                          // q rows of the group as A fragments
-  int cb = -1, cg = -1;                       // the (b, g) being accumulated
+  int cb = -1, cg = -1, cu = -1;              // the (b, g) being accumulated and its unit
   const int per = (total + nwarps - 1) / nwarps;
 
   auto reset = [&](int b, int g) {
@@ -219,8 +232,8 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   // write the current (b, g): the output itself when this segment holds all
   // of its batches, else a partial for the combine kernel
   auto flush = [&]() {
-    const int nb_ = s_nbat[cb];
-    const int firstb = s_bstart[cb] + cg * nb_;   // first batch of (cb, cg) in the list
+    const int nb_ = s_nbat[cu];
+    const int firstb = s_bstart[cu] + (a.kvh ? 0 : cg * nb_);   // first batch of (cb, cg) in the list
     const bool whole = firstb / per == (firstb + nb_ - 1) / per;   // one segment holds it all
     const int seg = gw - firstb / per;
     // (max, sum) of the heads in this lane's O^T columns
@@ -263,6 +276,7 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
       if (cb >= 0) flush();
       cb = pc.b;
       cg = pc.g;
+      cu = pc.u;
       reset(cb, cg);
     }
     // batch t is complete once at most min(kNS - 1, t1 - 1 - t) later groups are pending
@@ -384,14 +398,18 @@ __global__ void __launch_bounds__(kHeadDim) hill_attn_combine_kernel(AttnArgs a,
   pdl_wait();
   pdl_launch_dependents();
   if (dd == 0) {
+    // the batch layout of the attention kernel (see its table units)
+    const int R = a.kvh ? a.B * a.Hkv : a.B;
+    const int upb = a.kvh ? 1 : a.Hkv;
+    const int mine = a.kvh ? b * a.Hkv + g : b;
     int acc = 0, first = 0, nb = 0;
-    for (int bb = 0; bb < a.B; ++bb) {
-      const int nbb = (clamp_count(a, bb) + kBatch - 1) / kBatch;
-      if (bb == b) {
-        first = acc + g * nbb;
-        nb = nbb;
+    for (int u = 0; u < R; ++u) {
+      const int nbu = (clamp_count(a, u) + kBatch - 1) / kBatch;
+      if (u == mine) {
+        first = acc + (a.kvh ? 0 : g * nbu);
+        nb = nbu;
       }
-      acc += a.Hkv * nbb;
+      acc += upb * nbu;
     }
     s_first = first;
     s_nb = nb;

@@ -27,6 +27,7 @@ struct ScoreArgs {
   float* logits;      // ATTN: [B][H][cap]
   float2* partials;   // ATTN: [B][nslot][H] (max, sum 2^(z2 - max)), base-2 logits z2 = z * log2 e
   int nslot;          // = grid size of the launch
+  int kvh;            // RAW with per-KV-head selection: scores/accum [B][Hkv][cap], summed over each group only
   uint32_t* hist0;    // optional: zero-filled here (hist0_words words) for the normalisation to count into
   int64_t hist0_words;
   unsigned* err;
@@ -41,6 +42,8 @@ struct FinalizeArgs {
   float* accum;       // may be NULL
   uint32_t* hist0;    // optional [B][2048]: counts of the leading 11-bit digit of the selection key
   int recent;         // tokens j >= len - min(recent, len) are left out of hist0 (pinned, not ranked)
+  int kvh;            // 1: scores/accum are [B][Hkv][cap], the sum over each KV head's G query heads
+  int Hkv;
 };
 
 struct QuantArgs {
@@ -60,6 +63,7 @@ struct SelectArgs {
   int B, cap, max_k;
   int chunk;          // filled by the launcher
   const uint32_t* hist0;   // optional [B][2048]: counts of the leading 11-bit key digit (tokens j < len - recent)
+  int rows_per_seq;   // key rows per sequence: 1, or Hkv with per-KV-head selection (row r reads lens/k of r / rows_per_seq)
   int recent;         // BKP: the most recent min(recent, len) tokens are kept outright (0: none)
   uint16_t* hits;     // BKP: optional [B][cap] hit-rate table, +1 (saturating) per kept token
   int32_t* idx;
@@ -78,6 +82,7 @@ struct AttnArgs {
   float* out;         // [B][H][d]
   float* part;        // [B*H][splits][2 + d] partials of split (b, g) pairs
   int splits;         // partial slots per (b, h)
+  int kvh;            // 0: idx [B][max_k], count [B] shared by the KV heads; 1: idx [B][Hkv][max_k], count [B][Hkv]
   unsigned* err;
 };
 

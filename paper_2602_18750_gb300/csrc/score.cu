@@ -378,7 +378,18 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
           if constexpr (G >= 2) v += acc[mb][e + 1];
           if constexpr (G >= 4) v += __shfl_xor_sync(0xffffffffu, v, 1);
           if constexpr (G >= 8) v += __shfl_xor_sync(0xffffffffu, v, 2);
-          rs[u] += v;   // complete in the tig == 0 lanes
+          // complete in the tig == 0 lanes
+          if (a.kvh) {   // per-KV-head importance: this group's sum is the score of (b, g)
+            const int t = mb * 16 + grp + (u & 1) * 8;
+            if (tig == 0 && t < nv) {
+              const int64_t o = ((int64_t)b * Hkv + g) * cap + j0 + t;
+              const float val = v * kInvSqrtD;
+              if (a.scores) a.scores[o] = val;
+              if (a.accum) a.accum[o] += val;
+            }
+          } else {
+            rs[u] += v;
+          }
         }
       } else {
         float* lg = a.logits + ((int64_t)b * H + g * G) * cap + j0;
@@ -400,7 +411,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
         }
       }
     }
-    if (RAW) {
+    if (RAW && !a.kvh) {
       // sum over the warps in a fixed order, double-buffered by item; a warp
       // whose wait timed out still reaches the barrier, and all warps then
       // leave together
@@ -523,7 +534,40 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   if (a.hist0)
     for (int i = threadIdx.x; i < kHistBins; i += kFinThreads) hcount[i] = 0u;
   __syncthreads();
-  if (valid) {
+  if (valid && a.kvh) {
+    // per-KV-head importance: the sum over each group of G query heads,
+    // stored as soon as the group is complete (heads of a group are adjacent)
+    const int gm = a.H / a.Hkv - 1;   // G - 1 (G is a power of two)
+    auto put = [&](int g, float v) {
+      const int64_t o = ((int64_t)b * a.Hkv + g) * a.cap + j;
+      if (a.scores) a.scores[o] = v;
+      if (a.accum) a.accum[o] += v;
+    };
+    float sg = 0.f;
+#pragma unroll
+    for (int u = 0; u < kFinZReg; ++u)
+      if (u < a.H) {
+        sg += ex2(zr[u] - mh[u]) * il[u];
+        if (((u + 1) & gm) == 0) {
+          put(u / (gm + 1), sg);
+          sg = 0.f;
+        }
+      }
+    for (int h = kFinZReg; h < a.H; h += 16) {
+      float z[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) z[u] = h + u < a.H ? zp[(int64_t)(h + u) * a.cap] : 0.f;
+#pragma unroll
+      for (int u = 0; u < 16; ++u)
+        if (h + u < a.H) {
+          sg += ex2(z[u] - mh[h + u]) * il[h + u];
+          if (((h + u + 1) & gm) == 0) {
+            put((h + u) / (gm + 1), sg);
+            sg = 0.f;
+          }
+        }
+    }
+  } else if (valid) {
     float s = 0.f;
 #pragma unroll
     for (int u = 0; u < kFinZReg; ++u)

@@ -54,7 +54,10 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
   auto remote = [&](uint32_t* p, int c) -> uint32_t* {
     return CL ? cluster.map_shared_rank(p, c) : p;
   };
-  const int b = blockIdx.y;
+  // row = one key row; with per-KV-head selection a sequence has
+  // rows_per_seq rows that share its length and budget
+  const int row = blockIdx.y;
+  const int b = row / a.rows_per_seq;
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
   pdl_wait();
@@ -73,7 +76,7 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
   // never counted.
   const int j_lo = r * a.chunk;
   const int ncap = max(0, min(a.chunk, a.cap - j_lo));
-  const float* kp = a.key + (int64_t)b * a.cap + j_lo;
+  const float* kp = a.key + (int64_t)row * a.cap + j_lo;
 #pragma unroll 8
   for (int i = tid; i < ncap; i += kSelThreads) keys[i] = ordered_key(kp[i]);
   for (int i = tid; i < kHistBufs * kBins; i += kSelThreads) histbuf[i] = 0;
@@ -93,8 +96,8 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
     win = min(win, a.max_k);           // the most recent max_k tokens of the window
     kk = min(kk, a.max_k - win);
   }
-  int32_t* out = a.idx + (int64_t)b * a.max_k;
-  uint16_t* hits = a.hits ? a.hits + (int64_t)b * a.cap : nullptr;
+  int32_t* out = a.idx + (int64_t)row * a.max_k;
+  uint16_t* hits = a.hits ? a.hits + (int64_t)row * a.cap : nullptr;
   auto hit = [&](int j) {   // the hit-rate table: +1 per kept token, saturating
     if (hits && hits[j] != 0xffffu) hits[j] = (uint16_t)(hits[j] + 1u);
   };
@@ -102,7 +105,7 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
 
   // padding, count and the pinned window (every path)
   for (int p = kk + win + r * kSelThreads + tid; p < a.max_k; p += C * kSelThreads) out[p] = -1;
-  if (r == 0 && tid == 0) a.count[b] = kk + win;
+  if (r == 0 && tid == 0) a.count[row] = kk + win;
   for (int j = max(j_lo, len - win) + tid; j < min(j_lo + a.chunk, len); j += kSelThreads) {
     out[kk + j - (len - win)] = j;
     hit(j);
@@ -129,7 +132,7 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
     const uint32_t* om = merged;
     if (pass == 0 && a.hist0) {
       // leading-digit counts over the whole sequence, accumulated upstream
-      const uint32_t* h0 = a.hist0 + (int64_t)b * kBins;
+      const uint32_t* h0 = a.hist0 + (int64_t)row * kBins;
       for (int i = tid; i < kBins; i += kSelThreads) merged[i] = h0[i];
     } else {
       for (int i = tid; i < n; i += kSelThreads) {
@@ -292,7 +295,7 @@ cudaError_t launch_select(const SelectArgs& a0, cudaStream_t st) {
   const int C = select_cluster_size(a.cap);
   a.chunk = (a.cap + C - 1) / C;
   const size_t smem = select_smem_bytes(a.cap, C);
-  const dim3 grid(C, a.B, 1), block(kSelThreads, 1, 1);
+  const dim3 grid(C, a.B * a.rows_per_seq, 1), block(kSelThreads, 1, 1);
   if (C == 1) {
     static int cache[64] = {0};
     cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(hill_select_kernel<false>), (int)smem, cache);

@@ -9,6 +9,7 @@ fails loudly if the library has not been built.
 Names follow the C ABI: :func:`hill_score`, :func:`hill_topk_select`,
 :func:`hill_gather_sparse_attn`, :func:`hill_evict_step`, :func:`hill_topk_select_bkp`,
 :func:`hill_evict_step_bkp`, :func:`hill_quantize_k`, :func:`hill_score_f8`, :func:`hill_evict_step_f8`,
+:func:`hill_evict_step_kvh`,
 :func:`hill_workspace_bytes`, :func:`hill_sync_status`.
 """
 from __future__ import annotations
@@ -74,6 +75,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_topk_select_bkp.argtypes = [D, P, P, P, I32, I32, P, P, P, P, SZ, P]
     lib.hill_evict_step_bkp.argtypes = [D, P, P, P, P, P, I32, I32, I32, P, P, P, P, P, P, P, SZ, P]
     lib.hill_quantize_k.argtypes = [D, P, P, P, I32, P, P, P]
+    lib.hill_evict_step_kvh.argtypes = [D, P, P, P, P, P, I32, I32, P, P, P, P, P, P, SZ, P]
     lib.hill_score_f8.argtypes = [D, P, P, P, P, I32, P, P, P, SZ, P]
     lib.hill_evict_step_f8.argtypes = [D, P, P, P, P, P, P, P, I32, I32, P, P, P, P, P, P, SZ, P]
     lib.hill_score_noalloc.argtypes = [D, P, P, P, I32, P, P, P]
@@ -85,7 +87,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_kernel_launches.restype = ctypes.c_uint64
     for name in ("hill_score", "hill_topk_select", "hill_gather_sparse_attn", "hill_evict_step",
                  "hill_topk_select_bkp", "hill_evict_step_bkp", "hill_quantize_k", "hill_score_f8",
-                 "hill_evict_step_f8", "hill_sync_status"):
+                 "hill_evict_step_f8", "hill_evict_step_kvh", "hill_sync_status"):
         getattr(lib, name).restype = I32
     _lib = lib
     return lib
@@ -206,6 +208,15 @@ def hill_evict_step_bkp(desc, q, k_cache, v_cache, lens, k, recent, max_k, mode,
                                       _ptr(k), int(recent), int(max_k), int(mode), _ptr(accum), _ptr(scores),
                                       _ptr(idx), _ptr(count), _ptr(hits), _ptr(out), wp, wn,
                                       _stream(stream)), "hill_evict_step_bkp")
+
+
+def hill_evict_step_kvh(desc, q, k_cache, v_cache, lens, k, max_k, mode, accum, scores, idx, count, out, ws,
+                        stream=None) -> None:
+    """Per-KV-head selection: scores [B][Hkv][cap], idx [B][Hkv][max_k], count [B][Hkv]."""
+    wp, wn = _ws(ws)
+    _check(load().hill_evict_step_kvh(ctypes.byref(desc), _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(lens),
+                                      _ptr(k), int(max_k), int(mode), _ptr(accum), _ptr(scores), _ptr(idx),
+                                      _ptr(count), _ptr(out), wp, wn, _stream(stream)), "hill_evict_step_kvh")
 
 
 def shadow_shape(desc):

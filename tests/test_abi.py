@@ -30,7 +30,7 @@ def test_header_declares_the_boundary():
     names = _declared()
     for n in ("hill_score", "hill_topk_select", "hill_gather_sparse_attn", "hill_evict_step",
               "hill_topk_select_bkp", "hill_evict_step_bkp", "hill_quantize_k", "hill_score_f8",
-              "hill_evict_step_f8",
+              "hill_evict_step_f8", "hill_evict_step_kvh",
               "hill_workspace_bytes", "hill_sync_status", "hill_status_string", "hill_abi_version"):
         assert n in names
 
@@ -104,6 +104,12 @@ def test_host_validation_without_device(lib):
                              None) == INV
     assert lib.hill_evict_step_f8(ctypes.byref(d), FAKE, FAKE, None, None, None, FAKE, FAKE, 8, 0, None, None,
                                   FAKE, FAKE, None, FAKE, 1 << 30, None) == INV
+    # per-KV-head step: needs a score or accum buffer; B * Hkv above the attention table is unsupported
+    assert lib.hill_evict_step_kvh(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, 8, 0, None, None, FAKE, FAKE,
+                                   None, FAKE, 1 << 30, None) == INV
+    big = _desc(batch=100, num_q_heads=32, num_kv_heads=8, q_sb=32 * 128)
+    assert lib.hill_evict_step_kvh(ctypes.byref(big), FAKE, FAKE, FAKE, FAKE, FAKE, 8, 0, None, FAKE, FAKE, FAKE,
+                                   None, FAKE, 1 << 30, None) == UNS
     # BKP: a negative window is rejected before any device work
     assert lib.hill_topk_select_bkp(ctypes.byref(d), FAKE, FAKE, FAKE, -1, 8, FAKE, FAKE, None, None, 0,
                                     None) == INV
