@@ -292,9 +292,33 @@ def run_ours(args):
             hill.hill_evict_step(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], max_k, mode, acc,
                                  scores[l], idx[l], count[l], o, ws, st)
 
+    if args.overlap:
+        # layer-pipelined schedule (the APP analogue, Sec. 4.3): the evaluation
+        # and selection of layer l + 1 run on the main stream while the sparse
+        # attention of layer l runs on a side stream after its selection; the
+        # two phases use separate workspaces
+        side = torch.cuda.Stream(device=dev)
+        ws_attn = hill.alloc_workspace(desc, mode, max_k, dev)
+
     def issue_step(t, st):
+        if not args.overlap:
+            for l in range(L):
+                evict(t, l, out[l], st)
+            return
+        fork = torch.cuda.Event()
+        fork.record(st)
+        side.wait_event(fork)
         for l in range(L):
-            evict(t, l, out[l], st)
+            r = l % lres
+            evict(t, l, None, st)                       # evaluation + selection of layer l
+            sel = torch.cuda.Event()
+            sel.record(st)
+            side.wait_event(sel)
+            hill.hill_gather_sparse_attn(desc, q_all[t, l], Kall[r], Vall[r], idx[l], count[l], max_k, out[l],
+                                         ws_attn, side)
+        join = torch.cuda.Event()
+        join.record(side)
+        st.wait_event(join)
 
     # eager warm-up of every kernel shape, then one CUDA graph per decode step
     with torch.cuda.stream(stream):
@@ -440,7 +464,9 @@ def run_ours(args):
             "scaling": "weak", "vs_baseline": None, "dtype": "f16" if w.dtype == torch.float16 else "bf16",
             "data": "synthetic", "config": dict(describe(w, lres, args.mode),
                                                 **({"bkp_recent": args.bkp_recent} if bkp else {}),
-                                                **({"scoring": "e4m3 key shadow"} if f8 else {})),
+                                                **({"scoring": "e4m3 key shadow"} if f8 else {}),
+                                                **({"schedule": "layer-pipelined (2 streams)"} if args.overlap
+                                                   else {})),
             "k_stream_gbs": round(k_gbs, 1),
             "k_stream_frac_of_measured_hbm": round(k_gbs / world / peak, 4),
             "k_stream_frac_of_8tbs": round(k_gbs / world / 8000.0, 4),
@@ -611,6 +637,9 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--overlap", action="store_true",
+                    help="layer-pipelined schedule: attention of layer l on a second stream, overlapping the "
+                         "evaluation of layer l+1")
     ap.add_argument("--f8", action="store_true",
                     help="asymmetric-precision scoring (Sec. 4.4) from an E4M3 key shadow (hill_evict_step_f8)")
     ap.add_argument("--bkp-recent", type=int, default=-1,
