@@ -245,6 +245,13 @@ hill_status hill_score_noalloc(const hill_desc* desc, const void* q, const void*
  * caller count the kernels one call or one captured graph contains. */
 uint64_t hill_kernel_launches(void);
 
+/* Self-test of the bounded waits every kernel uses (no counterpart in the
+ * paper): launches one warp that waits on a barrier nothing will complete,
+ * for limit_us microseconds (1 .. 1e6), then gives up.  The wait expiring is
+ * recorded like any other: the next hill_sync_status() returns
+ * HILL_ERR_TIMEOUT, and the stream and context stay usable. */
+hill_status hill_selftest_wait(uint32_t limit_us, void* stream);
+
 /* ABI version of this header (major * 100 + minor). */
 int32_t hill_abi_version(void);
 

@@ -532,6 +532,13 @@ hill_status hill_evict_step_f8(const hill_desc* desc, const void* q, const uint8
                     ws, ws_bytes, stream, k8, kscale);
 }
 
+hill_status hill_selftest_wait(uint32_t limit_us, void* stream) {
+  if (limit_us == 0 || limit_us > 1000000u) return HILL_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  return from_cuda(counted(launch_selftest_wait(1000ull * limit_us, di.err, static_cast<cudaStream_t>(stream)), 1));
+}
+
 hill_status hill_sync_status(void* stream) {
   DeviceInfo di;
   if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;

@@ -141,6 +141,9 @@ int score_max_kv_heads(int G);
 cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8, int grid, cudaStream_t st);
 cudaError_t launch_attn_finalize(const FinalizeArgs& a, cudaStream_t st);
 
+// selftest.cu
+cudaError_t launch_selftest_wait(unsigned long long limit_ns, unsigned* err, cudaStream_t st);
+
 // quant.cu
 cudaError_t launch_quantize_k(const QuantArgs& a, int dtype, int max_rows, cudaStream_t st);
 

@@ -76,6 +76,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_evict_step_bkp.argtypes = [D, P, P, P, P, P, I32, I32, I32, P, P, P, P, P, P, P, SZ, P]
     lib.hill_quantize_k.argtypes = [D, P, P, P, I32, P, P, P]
     lib.hill_evict_step_kvh.argtypes = [D, P, P, P, P, P, I32, I32, P, P, P, P, P, P, SZ, P]
+    lib.hill_selftest_wait.argtypes = [ctypes.c_uint32, P]
     lib.hill_score_f8.argtypes = [D, P, P, P, P, I32, P, P, P, SZ, P]
     lib.hill_evict_step_f8.argtypes = [D, P, P, P, P, P, P, P, I32, I32, P, P, P, P, P, P, SZ, P]
     lib.hill_score_noalloc.argtypes = [D, P, P, P, I32, P, P, P]
@@ -87,7 +88,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_kernel_launches.restype = ctypes.c_uint64
     for name in ("hill_score", "hill_topk_select", "hill_gather_sparse_attn", "hill_evict_step",
                  "hill_topk_select_bkp", "hill_evict_step_bkp", "hill_quantize_k", "hill_score_f8",
-                 "hill_evict_step_f8", "hill_evict_step_kvh", "hill_sync_status"):
+                 "hill_evict_step_f8", "hill_evict_step_kvh", "hill_selftest_wait", "hill_sync_status"):
         getattr(lib, name).restype = I32
     _lib = lib
     return lib
@@ -249,6 +250,11 @@ def hill_evict_step_f8(desc, q, k8, kscale, k_cache, v_cache, lens, k, max_k, mo
                                      _ptr(v_cache), _ptr(lens), _ptr(k), int(max_k), int(mode), _ptr(accum),
                                      _ptr(scores), _ptr(idx), _ptr(count), _ptr(out), wp, wn, _stream(stream)),
            "hill_evict_step_f8")
+
+
+def hill_selftest_wait(limit_us: int, stream=None) -> None:
+    """Run the bounded-wait self test (its expiry shows up in hill_sync_status)."""
+    _check(load().hill_selftest_wait(int(limit_us), _stream(stream)), "hill_selftest_wait")
 
 
 def hill_kernel_launches() -> int:

@@ -30,7 +30,7 @@ def test_header_declares_the_boundary():
     names = _declared()
     for n in ("hill_score", "hill_topk_select", "hill_gather_sparse_attn", "hill_evict_step",
               "hill_topk_select_bkp", "hill_evict_step_bkp", "hill_quantize_k", "hill_score_f8",
-              "hill_evict_step_f8", "hill_evict_step_kvh",
+              "hill_evict_step_f8", "hill_evict_step_kvh", "hill_selftest_wait",
               "hill_workspace_bytes", "hill_sync_status", "hill_status_string", "hill_abi_version"):
         assert n in names
 
