@@ -33,7 +33,6 @@ namespace {
 
 constexpr int kAW = 8;                               // warps per CTA
 constexpr int kAThreads = kAW * 32;
-constexpr int kNS = 1;                               // shared-memory slots (batches in flight) per warp
 constexpr int kBatch = 32;                           // selected entries per batch
 constexpr int kMaxBatchAttn = 512;                   // sequences in the per-CTA table
 
@@ -42,7 +41,7 @@ constexpr int kHalfBytes = kBatch * 128;             // 32 rows x 64 dims, swizz
 struct AttnCfg {
   // K dims 0-63 | K dims 64-127 | V dims 0-63 | V dims 64-127
   static constexpr int kSlotBytes = 4 * kHalfBytes;
-  static constexpr int kSmem = kAW * kNS * kSlotBytes + 128;   // + alignment slack
+  static constexpr int kSmem = kAW * kSlotBytes + 128;   // + alignment slack
 };
 
 // Position of a batch in the list: table unit u (a sequence b, or with
@@ -103,8 +102,8 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   if (t0 >= t1) return;
 
   // 128-byte aligned slots: every swizzled row is one bank-aligned line
-  const uint32_t slot0 = ((smem_addr(asmem) + 127u) & ~127u) + warp * kNS * AttnCfg::kSlotBytes;
-  __shared__ unsigned s_vm[kAW][kNS];   // per slot: which rows of its batch hold a token
+  const uint32_t slot0 = ((smem_addr(asmem) + 127u) & ~127u) + warp * AttnCfg::kSlotBytes;
+  const uint32_t sk = slot0, sv = slot0 + 2 * kHalfBytes;   // the warp's K rows | V rows
   const auto* kbase = static_cast<const uint16_t*>(a.k);
   const auto* vbase = static_cast<const uint16_t*>(a.v);
   const int ksn = (int)a.k_sn, vsn = (int)a.v_sn;   // the host checks both fit in 32 bits
@@ -148,22 +147,27 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
     const int e = p.bi * kBatch + lane;
     return e < s_cnt[p.u] ? a.idx[(int64_t)p.u * a.max_k + e] : -1;
   };
-  // gather the batch at p into slot s: row r of the batch is token jj of
-  // lane r (-1: none, zero-filled).  A half-warp copies one 256-byte row;
-  // chunk c (16 bytes) of row r goes to 128-byte line r of half c / 8 at
-  // position (c % 8) ^ (r % 8), so the ldmatrix reads below are conflict-free.
+  // An entry of the batch at p that lies outside [0, cap) is reported and
+  // skipped (-1: no token).
+  auto check = [&](const Pos& p, int jj) -> int {
+    if (p.bi * kBatch + lane < s_cnt[p.u] && (jj < 0 || jj >= a.cap)) {
+      raise_error(a.err, kErrDevArg);
+      jj = -1;
+    }
+    return jj;
+  };
+  // Gather the 32 rows of one cache (K or V) for the batch at p into the
+  // 8 KB region dst: row r of the batch is token jj of lane r (-1: none,
+  // zero-filled).  A half-warp copies one 256-byte row; chunk c (16 bytes)
+  // of row r goes to 128-byte line r of half c / 8 at position
+  // (c % 8) ^ (r % 8), so the ldmatrix reads below are conflict-free.  One
+  // cp.async group per call.
   const int l16 = lane & 15, hrow = lane >> 4;
   const uint32_t dst_lane = (uint32_t)((l16 >> 3) * kHalfBytes + hrow * 128);
   const uint32_t swz_lane = (uint32_t)(((l16 & 7) ^ hrow) << 4);
-  auto issue = [&](const Pos& p, int s, int jj) -> unsigned {
-    if (p.bi * kBatch + lane < s_cnt[p.u] && (jj < 0 || jj >= a.cap)) {
-      raise_error(a.err, kErrDevArg);   // a listed entry outside [0, cap): skipped
-      jj = -1;
-    }
-    const unsigned vm = __ballot_sync(0xffffffffu, jj >= 0);
-    const uint32_t sk = slot0 + s * AttnCfg::kSlotBytes + dst_lane;
-    const uint16_t* kr = kbase + (int64_t)p.b * a.k_sb + (int64_t)p.g * a.k_sh + l16 * 8;
-    const uint16_t* vr = vbase + (int64_t)p.b * a.v_sb + (int64_t)p.g * a.v_sh + l16 * 8;
+  auto issue_rows = [&](const Pos& p, uint32_t dst, const uint16_t* base, int64_t sb, int64_t sh, int sn, int jj) {
+    const uint16_t* rp = base + (int64_t)p.b * sb + (int64_t)p.g * sh + l16 * 8;
+    dst += dst_lane;
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
       const int j = __shfl_sync(0xffffffffu, jj, 2 * i + hrow);
@@ -171,34 +175,26 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
       const int jc = j >= 0 ? j : 0;
       // row 2i + hrow: (2i + hrow) % 8 = (2i % 8) | hrow
       const uint32_t off = (uint32_t)(i * 256) + (swz_lane ^ (uint32_t)(((2 * i) & 7) << 4));
-      cp_async16_zfill(sk + off, kr + (int64_t)jc * ksn, nbytes);
-      cp_async16_zfill(sk + 2 * kHalfBytes + off, vr + (int64_t)jc * vsn, nbytes);
+      cp_async16_zfill(dst + off, rp + (int64_t)jc * sn, nbytes);
     }
     cp_async_commit();
-    return vm;
   };
 
-  // prologue: batches t0 .. t0 + kNS - 1, and the indices of t0 + kNS
+  // Pipeline of one warp over its batches t0 .. t1-1, with one K region and
+  // one V region: K rows of batch t + 1 are fetched once S(t) has read the K
+  // region (while the softmax and O += P V of batch t run), V rows of batch
+  // t + 1 once O += P V(t) has read the V region (while S(t + 1) runs).  The
+  // cp.async groups complete in the order K(t), V(t), K(t + 1), V(t + 1), ...
+  // The index entries of batch t + 2 are loaded when K(t + 1) is issued.
   Pos pc = first, pi = first, pl = first;
-  int jnext = -1;
-  {
-    int jq[kNS];
-#pragma unroll
-    for (int u = 0; u < kNS; ++u) {
-      jq[u] = t0 + u < t1 ? load_idx(pl) : -1;
-      advance(pl);
-    }
-#pragma unroll
-    for (int u = 0; u < kNS; ++u) {
-      if (t0 + u < t1) {
-        const unsigned v = issue(pi, u, jq[u]);
-        if (lane == 0) s_vm[warp][u] = v;
-        advance(pi);
-      }
-    }
-    if (t0 + kNS < t1) jnext = load_idx(pl);
-    advance(pl);
-  }
+  int jcur = check(pi, load_idx(pl));           // entries of the batch being issued
+  advance(pl);
+  unsigned vm_cur = __ballot_sync(0xffffffffu, jcur >= 0), vm_next = 0u;
+  issue_rows(pi, sk, kbase, a.k_sb, a.k_sh, ksn, jcur);
+  issue_rows(pi, sv, vbase, a.v_sb, a.v_sh, vsn, jcur);
+  advance(pi);
+  int jnext = t0 + 1 < t1 ? load_idx(pl) : -1;
+  advance(pl);
 
   // mma.sync fragments: grp = lane/4, tig = lane%4.  S accumulators: row grp
   // = query head grp of the group (rows >= G and 8..15 are zero), columns =
@@ -269,9 +265,6 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   };
 
   for (int t = t0; t < t1; ++t) {
-    const int s = (t - t0) % kNS;
-    const uint32_t sk = slot0 + s * AttnCfg::kSlotBytes;
-    const uint32_t sv = sk + 2 * kHalfBytes;
     if (pc.b != cb || pc.g != cg) {
       if (cb >= 0) flush();
       cb = pc.b;
@@ -279,14 +272,11 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
       cu = pc.u;
       reset(cb, cg);
     }
-    // batch t is complete once at most min(kNS - 1, t1 - 1 - t) later groups are pending
-    const int later = min(kNS - 1, t1 - 1 - t);
-    if (later >= kNS - 1) cp_async_wait<kNS - 1>();
-    else if (kNS > 2 && later == 2) cp_async_wait<(kNS > 2 ? 2 : 0)>();
-    else if (later == 1) cp_async_wait<1>();
-    else cp_async_wait<0>();
+    // K(t) is complete once at most V(t) is pending
+    cp_async_wait<1>();
     __syncwarp();
-    const unsigned vm = s_vm[warp][s];
+    const unsigned vm = vm_cur;
+    const bool more = t + 1 < t1;
 
     // S = q . K^T: A = q (16 rows = heads), B = K rows (n = 8 tokens)
     float sacc[4][4];
@@ -305,6 +295,15 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
         mma_16816<DT>(sacc[nb], a0, bk[0], bk[1]);
         mma_16816<DT>(sacc[nb], a1, bk[2], bk[3]);
       }
+    }
+    // the K region is free: fetch K(t + 1), and the entries of batch t + 2
+    __syncwarp();
+    if (more) {
+      jcur = check(pi, jnext);
+      vm_next = __ballot_sync(0xffffffffu, jcur >= 0);
+      issue_rows(pi, sk, kbase, a.k_sb, a.k_sh, ksn, jcur);
+      jnext = t + 2 < t1 ? load_idx(pl) : -1;
+      advance(pl);
     }
     // online softmax of head grp over the batch's tokens nb*8 + 2*tig + {0,1}
     float z[8];
@@ -357,6 +356,10 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
         pb[kt][0][hf] = hi;
         pb[kt][1][hf] = pack2<DT>(x - hv.x, y - hv.y);
       }
+    // V(t) is complete once at most K(t + 1) is pending
+    if (more) cp_async_wait<1>();
+    else cp_async_wait<0>();
+    __syncwarp();
     // O^T += V^T . P^T: A = V^T (16 dims x 16 tokens) by transposed ldmatrix
 #pragma unroll
     for (int kt = 0; kt < 2; ++kt) {
@@ -370,15 +373,13 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
         mma_16816<DT>(oacc[db], av, pb[kt][1][0], pb[kt][1][1]);
       }
     }
-    // the slot is free: refill it with batch t + kNS, prefetch the indices of t + kNS + 1
+    // the V region is free: fetch V(t + 1)
     __syncwarp();
-    if (t + kNS < t1) {
-      const unsigned v = issue(pi, s, jnext);
-      if (lane == 0) s_vm[warp][s] = v;
+    if (more) {
+      issue_rows(pi, sv, vbase, a.v_sb, a.v_sh, vsn, jcur);
       advance(pi);
-      jnext = t + kNS + 1 < t1 ? load_idx(pl) : -1;
-      advance(pl);
     }
+    vm_cur = vm_next;
     advance(pc);
   }
   flush();
@@ -386,25 +387,37 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
 
 // Merge the partials of one (b, h) whose batches were split over several
 // warps: out = sum_s 2^{M_s - M} O_s / sum_s 2^{M_s - M} L_s (maxima in the
-// base-2 scale of the attention kernel).  Pairs held
-// whole by one warp were written directly; sequences with no selected token
-// get zeros.
-__global__ void __launch_bounds__(kHeadDim) hill_attn_combine_kernel(AttnArgs a, int total_warps) {
+// base-2 scale of the attention kernel).  Pairs held whole by one warp were
+// written directly; sequences with no selected token get zeros.  One CTA per
+// (b, h): kCombGroups groups of kHeadDim threads (one per output dimension)
+// each merge every kCombGroups-th partial with a running maximum, the loads
+// of several partials in flight at once, and the group results are merged in
+// shared memory.  A short budget split over many warps (one batch per warp)
+// leaves dozens of partials per pair, so their loads must not be serialised.
+constexpr int kCombGroups = 4;
+constexpr int kCombThreads = kCombGroups * kHeadDim;
+
+__global__ void __launch_bounds__(kCombThreads) hill_attn_combine_kernel(AttnArgs a, int total_warps) {
   __shared__ int s_first, s_nb, s_total;
+  __shared__ float s_m[kCombGroups], s_l[kCombGroups];
+  __shared__ float s_o[kCombGroups][kHeadDim];
   const int bh = blockIdx.x;
   const int b = bh / a.H, h = bh % a.H;
   const int G = a.H / a.Hkv, g = h / G;
-  const int dd = threadIdx.x;
+  const int tid = threadIdx.x, dd = tid % kHeadDim, gi = tid / kHeadDim;
+  __shared__ int s_nbu[kMaxBatchAttn];
   pdl_wait();
   pdl_launch_dependents();
-  if (dd == 0) {
-    // the batch layout of the attention kernel (see its table units)
-    const int R = a.kvh ? a.B * a.Hkv : a.B;
+  // the batch layout of the attention kernel (see its table units)
+  const int R = a.kvh ? a.B * a.Hkv : a.B;
+  for (int u = tid; u < R; u += kCombThreads) s_nbu[u] = (clamp_count(a, u) + kBatch - 1) / kBatch;
+  __syncthreads();
+  if (tid == 0) {
     const int upb = a.kvh ? 1 : a.Hkv;
     const int mine = a.kvh ? b * a.Hkv + g : b;
     int acc = 0, first = 0, nb = 0;
     for (int u = 0; u < R; ++u) {
-      const int nbu = (clamp_count(a, u) + kBatch - 1) / kBatch;
+      const int nbu = s_nbu[u];
       if (u == mine) {
         first = acc + (a.kvh ? 0 : g * nbu);
         nb = nbu;
@@ -419,26 +432,58 @@ __global__ void __launch_bounds__(kHeadDim) hill_attn_combine_kernel(AttnArgs a,
   const int nb = s_nb, first = s_first, total = s_total;
   float* op = a.out + (int64_t)bh * kHeadDim + dd;
   if (nb == 0) {
-    *op = 0.f;
+    if (gi == 0) *op = 0.f;
     return;
   }
   const int per = (total + total_warps - 1) / total_warps;
   const int w0 = first / per, w1 = (first + nb - 1) / per;
   if (w0 == w1) return;   // one warp held every batch and wrote the output
-  const float* pp = a.part + (int64_t)bh * a.splits * (2 + kHeadDim);
+  constexpr int kPS = 2 + kHeadDim;   // one partial: max, sum, o[kHeadDim]
+  const float* pp = a.part + (int64_t)bh * a.splits * kPS;
   const int nseg = w1 - w0 + 1;
-  float M = -INFINITY;
-  for (int s = 0; s < nseg; ++s) M = fmaxf(M, pp[s * (2 + kHeadDim)]);
-  float L = 0.f, O = 0.f;
-  if (M != -INFINITY) {
-    for (int s = 0; s < nseg; ++s) {
-      const float* q = pp + s * (2 + kHeadDim);
-      const float c = ex2(q[0] - M);   // partial maxima are in the base-2 scale
-      L += q[1] * c;
-      O += q[2 + dd] * c;
+  float M = -INFINITY, L = 0.f, O = 0.f;
+  constexpr int kU = 16;  // partials per group whose loads are issued together
+  for (int s0 = gi; s0 < nseg; s0 += kCombGroups * kU) {
+    float ms[kU], ls[kU], os[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int s = s0 + u * kCombGroups;
+      const float* q = pp + (int64_t)s * kPS;
+      ms[u] = s < nseg ? q[0] : -INFINITY;
+      ls[u] = s < nseg ? q[1] : 0.f;
+      os[u] = s < nseg ? q[2 + dd] : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      if (ms[u] == -INFINITY) continue;   // past the end (every written partial holds a token)
+      const float mn = fmaxf(M, ms[u]);
+      const float c0 = ex2(M - mn), c1 = ex2(ms[u] - mn);   // partial maxima are in the base-2 scale
+      L = L * c0 + ls[u] * c1;
+      O = O * c0 + os[u] * c1;
+      M = mn;
     }
   }
-  *op = L > 0.f ? O / L : 0.f;
+  s_o[gi][dd] = O;
+  if (dd == 0) {
+    s_m[gi] = M;
+    s_l[gi] = L;
+  }
+  __syncthreads();
+  if (gi == 0) {
+    float Mx = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < kCombGroups; ++i) Mx = fmaxf(Mx, s_m[i]);
+    float Ls = 0.f, Os = 0.f;
+    if (Mx != -INFINITY) {
+#pragma unroll
+      for (int i = 0; i < kCombGroups; ++i) {
+        const float c = s_m[i] == -INFINITY ? 0.f : ex2(s_m[i] - Mx);
+        Ls += s_l[i] * c;
+        Os += s_o[i][dd] * c;
+      }
+    }
+    *op = Ls > 0.f ? Os / Ls : 0.f;
+  }
 }
 
 template <int DT, int G>
@@ -449,7 +494,7 @@ cudaError_t launch_attn_t(const AttnArgs& a, int grid, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   e = launch_pdl(kern, dim3(grid), dim3(kAThreads), AttnCfg::kSmem, st, 0, a);
   if (e != cudaSuccess) return e;
-  return launch_pdl(hill_attn_combine_kernel, dim3(a.B * a.H), dim3(kHeadDim), 0, st, 0, a, grid * kAW);
+  return launch_pdl(hill_attn_combine_kernel, dim3(a.B * a.H), dim3(kCombThreads), 0, st, 0, a, grid * kAW);
 }
 
 template <int DT>

@@ -462,21 +462,16 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   float* mh = fsm;            // [H]
   float* il = fsm + a.H;      // [H]
   uint32_t* hcount = reinterpret_cast<uint32_t*>(fsm + 2 * a.H);   // [kHistBins] when a.hist0
-  pdl_wait();
-  pdl_launch_dependents();
+  // The lengths are inputs of the call: this kernel only ever follows the
+  // scoring kernel of the same call, whose own dependency wait covered every
+  // earlier write, so they are read before this kernel's wait and overlap
+  // the end of the scoring kernel.  Everything the scoring kernel writes
+  // (logits, partials) is read after the wait.
   const int b = blockIdx.y;
   int len = a.lens[b];
   len = len < 0 ? 0 : (len > a.cap ? a.cap : len);
   const int jb = blockIdx.x * kFinChunk;
   if (jb >= len) return;
-  // this token's logits of the first kFinZReg heads, loaded before the
-  // partials are combined so that both round trips overlap
-  const int j = jb + threadIdx.x;
-  const bool valid = j < len;
-  const float* zp = a.logits + (int64_t)b * a.H * a.cap + j;
-  float zr[kFinZReg];
-#pragma unroll
-  for (int u = 0; u < kFinZReg; ++u) zr[u] = (valid && u < a.H) ? zp[(int64_t)u * a.cap] : 0.f;
   // the scoring CTAs that met b wrote slots 0 .. ns-1
   // (every thread counts the tiles of a share of the sequences)
   __shared__ int s_first, s_total;
@@ -499,6 +494,16 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   const int per = (s_total + a.nslot - 1) / a.nslot;
   const int items = (len + kT - 1) / kT;
   const int ns = (first_item + items - 1) / per - first_item / per + 1;
+  pdl_wait();
+  pdl_launch_dependents();
+  // this token's logits of the first kFinZReg heads, loaded before the
+  // partials are combined so that both round trips overlap
+  const int j = jb + threadIdx.x;
+  const bool valid = j < len;
+  const float* zp = a.logits + (int64_t)b * a.H * a.cap + j;
+  float zr[kFinZReg];
+#pragma unroll
+  for (int u = 0; u < kFinZReg; ++u) zr[u] = (valid && u < a.H) ? zp[(int64_t)u * a.cap] : 0.f;
   const float2* pb = a.partials + (int64_t)b * a.nslot * a.H;
   const int sub = threadIdx.x % kFinPartThreads;
   for (int h = threadIdx.x / kFinPartThreads; h < a.H; h += kFinThreads / kFinPartThreads) {

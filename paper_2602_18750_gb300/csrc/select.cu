@@ -38,6 +38,8 @@ constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kBins = 2048;
 constexpr int kMaxCluster = 8;
 constexpr int kChunkMax = 16384;   // keys per CTA before the cluster grows
+constexpr int kCand = kBins;       // crossing-bucket keys a cluster gathers into each CTA
+constexpr int kCandMinCluster = 8; // cluster size from which it gathers them
 constexpr int kHistBufs = 3;       // one per pass: no buffer is rewritten while a peer may read it
 
 template <bool CL>
@@ -63,25 +65,50 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
   pdl_wait();
   pdl_launch_dependents();
 
-  extern __shared__ uint32_t sm[];
+  extern __shared__ __align__(16) uint32_t sm[];
   uint32_t* keys = sm;                       // [chunk]
   uint32_t* histbuf = keys + a.chunk;        // [kHistBufs][kBins], pass p uses buffer p
   uint32_t* merged = histbuf + kHistBufs * kBins;   // [kBins]: the cluster's sum for this pass
   __shared__ uint32_t wtot[kSelWarps];
   __shared__ uint32_t cnt[kMaxCluster];
+  __shared__ uint32_t cnt2[kMaxCluster];
+  __shared__ uint32_t s_nc;
   __shared__ uint32_t bc[3];
 
-  // Load this CTA's chunk of keys before the lengths are known: every row
-  // below the capacity is valid memory, and rows at or beyond the length are
-  // never counted.
+  // Every global read the search needs is issued before the first use of
+  // any of them, so the kernel pays one memory round trip, not one per
+  // input: the length and budget, the upstream leading-digit histogram, and
+  // this CTA's chunk of keys.  The keys are read up to the capacity (valid
+  // memory); rows at or beyond the length are never counted.
+  int len = a.lens[b];
+  int kk = a.k[b];
+  constexpr int kH0 = kBins / kSelThreads;
+  uint32_t h0v[kH0];
+  if (a.hist0) {
+    const uint32_t* h0 = a.hist0 + (int64_t)row * kBins;
+#pragma unroll
+    for (int j = 0; j < kH0; ++j) h0v[j] = h0[tid + j * kSelThreads];
+  }
   const int j_lo = r * a.chunk;
   const int ncap = max(0, min(a.chunk, a.cap - j_lo));
   const float* kp = a.key + (int64_t)row * a.cap + j_lo;
+  int i_tail = 0;
+  if ((reinterpret_cast<uintptr_t>(kp) & 15u) == 0) {
+    // 16-byte loads when the chunk starts on a 16-byte boundary
+    const int n4 = ncap >> 2;
+    const float4* kp4 = reinterpret_cast<const float4*>(kp);
+    uint4* k4 = reinterpret_cast<uint4*>(keys);
+#pragma unroll 4
+    for (int i = tid; i < n4; i += kSelThreads) {
+      const float4 v = kp4[i];
+      k4[i] = make_uint4(ordered_key(v.x), ordered_key(v.y), ordered_key(v.z), ordered_key(v.w));
+    }
+    i_tail = n4 << 2;
+  }
 #pragma unroll 8
-  for (int i = tid; i < ncap; i += kSelThreads) keys[i] = ordered_key(kp[i]);
+  for (int i = i_tail + tid; i < ncap; i += kSelThreads) keys[i] = ordered_key(kp[i]);
   for (int i = tid; i < kHistBufs * kBins; i += kSelThreads) histbuf[i] = 0;
 
-  int len = a.lens[b];
   len = len < 0 ? 0 : (len > a.cap ? a.cap : len);
   // BKP temporal pinning (Sec. 4.2): the most recent tokens [older, len) are
   // kept outright; the ranking runs over [0, older)
@@ -89,7 +116,6 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
   const int rfull = rec < len ? rec : len;
   const int older = len - rfull;
   int win = rfull;
-  int kk = a.k[b];
   kk = kk < 0 ? 0 : (kk > older ? older : kk);
   if (win > a.max_k || kk > a.max_k - min(win, a.max_k)) {
     if (r == 0 && tid == 0) raise_error(a.err, kErrDevArg);
@@ -123,6 +149,9 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
   uint32_t prefix = 0, pmask = 0;
   uint32_t remaining = (uint32_t)kk;
   bool take_bucket = false;    // the crossing bucket is taken whole
+  const uint32_t* src = keys;  // the keys histogrammed by passes 1 and 2
+  int nsrc = n;
+  bool local = !CL;            // a pass needs no exchange between CTAs
 #pragma unroll 1
   for (int pass = 0; pass < 3; ++pass) {
     const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
@@ -132,23 +161,33 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
     const uint32_t* om = merged;
     if (pass == 0 && a.hist0) {
       // leading-digit counts over the whole sequence, accumulated upstream
-      const uint32_t* h0 = a.hist0 + (int64_t)row * kBins;
-      for (int i = tid; i < kBins; i += kSelThreads) merged[i] = h0[i];
+#pragma unroll
+      for (int j = 0; j < kH0; ++j) merged[tid + j * kSelThreads] = h0v[j];
     } else {
-      for (int i = tid; i < n; i += kSelThreads) {
-        const uint32_t kv = keys[i];
+      for (int i = tid; i < nsrc; i += kSelThreads) {
+        const uint32_t kv = src[i];
         if ((kv & pmask) == prefix) atomicAdd(&hist[(kv >> shift) & dmask], 1u);
       }
-      csync();  // every CTA's histogram of this pass is complete
-      if (CL) {
-        for (int i = tid; i < nb; i += kSelThreads) {
-          uint32_t v = 0;
-          for (int c = 0; c < C; ++c) v += remote(hist, c)[i];
-          merged[i] = v;
-        }
+      if (local) {
+        __syncthreads();
       } else {
-        om = hist;
+        csync();  // every CTA's histogram of this pass is complete
+        // all peer reads are issued before any sum is stored
+        uint32_t v[kH0] = {};
+#pragma unroll
+        for (int c = 0; c < kMaxCluster; ++c) {
+          if (c < C) {
+            const uint32_t* h = remote(hist, c);
+#pragma unroll
+            for (int j = 0; j < kH0; ++j)
+              if (tid + j * kSelThreads < nb) v[j] += h[tid + j * kSelThreads];
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < kH0; ++j)
+          if (tid + j * kSelThreads < nb) merged[tid + j * kSelThreads] = v[j];
       }
+      if (local) om = hist;
     }
     __syncthreads();
     // Two-level search over positions p = 0..nb-1 (bins from the top down):
@@ -203,6 +242,65 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
     if (remaining == bc[2]) {
       take_bucket = true;
       break;
+    }
+    if (!local && pass == 0 && C >= kCandMinCluster && bc[2] <= (uint32_t)kCand) {
+      // The keys of the crossing bucket are few (typically 1-4 % of the
+      // sequence): every CTA gathers all of them from the cluster once, and
+      // passes 1 and 2 then run on that copy inside each CTA, with no
+      // further histogram exchange.  All CTAs hold the same multiset, so
+      // they reach the same digits.  (Measured: this pays off against the
+      // exchange of 2 x C histograms at C = 8 and loses at C = 2.)  The buffers: this CTA's own candidates
+      // go to `merged` (free after the search above; peers read it until
+      // the compaction's cluster barrier), the gathered copy to histogram
+      // buffer 0 (peers have finished reading it once they pass the barrier
+      // below).
+      uint32_t* cand = merged;
+      if (tid == 0) s_nc = 0;
+      __syncthreads();
+      for (int w0 = warp * 32; w0 < n; w0 += kSelThreads) {   // warp-uniform trip count
+        const int i = w0 + lane;
+        const uint32_t kv = i < n ? keys[i] : 0u;
+        const bool m = i < n && (kv & pmask) == prefix;
+        const unsigned bal = __ballot_sync(0xffffffffu, m);
+        if (bal) {
+          uint32_t base = 0;
+          if (lane == 0) base = atomicAdd(&s_nc, (uint32_t)__popc(bal));
+          base = __shfl_sync(0xffffffffu, base, 0) + (uint32_t)__popc(bal & ((1u << lane) - 1u));
+          if (m && base < (uint32_t)kCand) cand[base] = kv;
+        }
+      }
+      __syncthreads();
+      if (tid < C) remote(cnt2, tid)[r] = s_nc;
+      csync();  // every CTA's candidates and count are in place
+      uint32_t offs[kMaxCluster + 1];
+      offs[0] = 0;
+#pragma unroll
+      for (int c = 0; c < kMaxCluster; ++c) offs[c + 1] = offs[c] + (c < C ? min(cnt2[c], (uint32_t)kCand) : 0u);
+      const uint32_t tot = offs[kMaxCluster];
+      if (tot != bc[2] && tid == 0) raise_error(a.err, kErrDevArg);   // cannot happen: counts disagree
+      uint32_t* all = histbuf;
+      constexpr int kCandPer = kCand / kSelThreads;
+      uint32_t v[kCandPer];
+#pragma unroll
+      for (int j = 0; j < kCandPer; ++j) {   // every peer read is issued before any store
+        const uint32_t i = (uint32_t)(tid + j * kSelThreads);
+        int c = 0;
+        uint32_t base = 0;
+#pragma unroll
+        for (int cc = 1; cc < kMaxCluster; ++cc)
+          if (i >= offs[cc]) {
+            c = cc;
+            base = offs[cc];
+          }
+        v[j] = i < tot ? remote(cand, c)[i - base] : 0u;
+      }
+#pragma unroll
+      for (int j = 0; j < kCandPer; ++j)
+        if ((uint32_t)(tid + j * kSelThreads) < tot) all[tid + j * kSelThreads] = v[j];
+      src = all;
+      nsrc = (int)min(tot, (uint32_t)kCand);
+      local = true;
+      __syncthreads();
     }
   }
   // Selection rule: take_bucket -> key >= prefix (every key of the crossing

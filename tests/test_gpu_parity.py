@@ -202,6 +202,34 @@ def test_topk_multi_cta_clusters(H, oracle_mod, cap):
     assert np.array_equal(cnt.cpu().numpy(), cnt_o)
 
 
+@pytest.mark.parametrize("cap", [40000, 131072 + 7])
+def test_topk_cluster_gathered_crossing_bucket(H, oracle_mod, cap):
+    """Log-normal scores spread over many octaves, so the bucket of the
+    leading 11 key bits that holds the k-th key is small and the cluster
+    finishes the search on a gathered copy of it; exact ties planted at the
+    k-th score exercise the lowest-index rule there."""
+    B = 3
+    g = torch.Generator().manual_seed(cap + 1)
+    s = torch.exp(torch.randn(B, cap, generator=g) * 4)
+    lens, k = [cap, cap - 977, cap // 3], [cap // 5, 3001, 517]
+    for b in range(B):
+        tau = torch.sort(s[b, : lens[b]], descending=True).values[k[b] - 1]
+        pos = torch.randint(0, lens[b], (9,), generator=g)
+        s[b, pos] = tau
+    q, K, V, lens_t = _case(B, 4, 4, 64, [64, 64, 64], torch.float16, seed=1)
+    desc = H.make_desc(q, K, V)
+    desc.capacity = cap
+    max_k = max(k)
+    idx = torch.empty(B, max_k, dtype=torch.int32, device="cuda")
+    cnt = torch.empty(B, dtype=torch.int32, device="cuda")
+    H.hill_topk_select(desc, s.cuda(), torch.tensor(lens, dtype=torch.int32, device="cuda"),
+                       torch.tensor(k, dtype=torch.int32, device="cuda"), max_k, idx, cnt)
+    H.hill_sync_status()
+    idx_o, cnt_o, _ = oracle_mod.topk(s.numpy().astype(np.float64), lens, k, max_k)
+    assert np.array_equal(idx.cpu().numpy(), idx_o)
+    assert np.array_equal(cnt.cpu().numpy(), cnt_o)
+
+
 def test_attention_full_budget_is_dense(H):
     """k = len: the sparse attention is the dense decode attention (checked
     against torch's SDPA on the GPU in float64)."""
