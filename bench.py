@@ -43,6 +43,8 @@ import torch  # noqa: E402
 from paper_2602_18750_gb300 import inputs  # noqa: E402
 
 METRIC = "cached tokens scored+selected/sec"
+# keyed by --serial
+SCHEDULES = {False: "layer-pipelined (2 streams, Sec. 4.3)", True: "serial (one fused hill_evict_step per layer)"}
 UNIT = "tokens/s"
 L2_BYTES = 129 * 1024 * 1024
 
@@ -292,16 +294,17 @@ def run_ours(args):
             hill.hill_evict_step(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], max_k, mode, acc,
                                  scores[l], idx[l], count[l], o, ws, st)
 
-    if args.overlap:
-        # layer-pipelined schedule (the APP analogue, Sec. 4.3): the evaluation
-        # and selection of layer l + 1 run on the main stream while the sparse
-        # attention of layer l runs on a side stream after its selection; the
-        # two phases use separate workspaces
-        side = torch.cuda.Stream(device=dev)
-        ws_attn = hill.alloc_workspace(desc, mode, max_k, dev)
+    # Layer-pipelined schedule (the APP analogue, Sec. 4.3; the default): the
+    # evaluation and selection of layer l + 1 run on the main stream while the
+    # sparse attention of layer l runs on a side stream after its selection;
+    # the two phases use separate workspaces.  The serial schedule runs one
+    # fused hill_evict_step per layer.  Both are timed; --serial makes the
+    # serial one the headline.
+    side = torch.cuda.Stream(device=dev)
+    ws_attn = hill.alloc_workspace(desc, mode, max_k, dev)
 
-    def issue_step(t, st):
-        if not args.overlap:
+    def issue_step(t, st, serial=args.serial):
+        if serial:
             for l in range(L):
                 evict(t, l, out[l], st)
             return
@@ -371,6 +374,36 @@ def run_ours(args):
     k_bytes_per_token = Hkv * (d + 4) if f8 else Hkv * d * 2
     k_gbs = world * tokens * k_bytes_per_token / (ms / 1e3) / 1e9
     gpu_launches = sum(launches[t] for t in order)
+
+    # ---------------- the other schedule, the same steps, timed the same way
+    other_graphs = []
+    for t in range(S):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            issue_step(t, stream, serial=not args.serial)
+        other_graphs.append(g)
+    if accum is not None:
+        accum.zero_()
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            other_graphs[i % S].replay()
+    barrier(dev)
+    torch.cuda.synchronize(dev)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for t in order:
+            other_graphs[t].replay()
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(dev)
+    ms_other = max_over_ranks(e0.elapsed_time(e1), dev)
+    hill.hill_sync_status(stream)
+    other_schedule = {
+        "schedule": SCHEDULES[not args.serial],
+        "us_per_layer": round(ms_other * 1e3 / (len(order) * L), 2),
+        "tokens_per_s": round(world * tokens / (ms_other / 1e3), 1),
+    }
+    del other_graphs
 
     # ---------------- evaluation + selection only (no attention): the same steps
     # with out = NULL, one graph per decode step, timed like the main region
@@ -451,7 +484,7 @@ def run_ours(args):
     e2e = None
     if not args.no_e2e:
         e2e = run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all, accum, scores,
-                      idx, count, out, ws, stream, dev, world)
+                      idx, count, out, ws, stream, dev, world, side, ws_attn)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -465,12 +498,12 @@ def run_ours(args):
             "data": "synthetic", "config": dict(describe(w, lres, args.mode),
                                                 **({"bkp_recent": args.bkp_recent} if bkp else {}),
                                                 **({"scoring": "e4m3 key shadow"} if f8 else {}),
-                                                **({"schedule": "layer-pipelined (2 streams)"} if args.overlap
-                                                   else {})),
+                                                schedule=SCHEDULES[args.serial]),
             "k_stream_gbs": round(k_gbs, 1),
             "k_stream_frac_of_measured_hbm": round(k_gbs / world / peak, 4),
             "k_stream_frac_of_8tbs": round(k_gbs / world / 8000.0, 4),
             "eval_step_us_per_layer": round(step_us_per_layer, 2),
+            "other_schedule": other_schedule,
             "eval_select": eval_select,
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": gpu_launches,
             "clocks": clock_info, "generate_s": round(t_gen, 1),
@@ -481,8 +514,11 @@ def run_ours(args):
 
 
 def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all, accum, scores, idx, count,
-            out, ws, stream, dev, world):
-    """Same steps through hill_evict_step (eager calls), with each step's inputs
+            out, ws, stream, dev, world, side, ws_attn):
+    """Same steps through the public calls (eager, in the bench's schedule:
+    hill_evict_step per layer, or with the layer-pipelined schedule
+    hill_evict_step without attention on the main stream and
+    hill_gather_sparse_attn on the side stream), with each step's inputs
     copied from pinned host memory (query of every layer, the new token's K/V
     row of every layer, lengths, budgets) and its results (selection and
     attention output of every layer) copied back, all inside the timed region."""
@@ -506,6 +542,14 @@ def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all,
     cnt_h = torch.empty_like(count, device="cpu").pin_memory()
     out_h = torch.empty_like(out, device="cpu").pin_memory()
     uniform = [len(set(p)) == 1 for p in pos]
+    # per-layer views and events, made once (as an engine would hold them)
+    qv = [[q_all[t, l] for l in range(L)] for t in range(S)]
+    Kv, Vv = [Kall[r] for r in range(lres)], [Vall[r] for r in range(lres)]
+    accv = [accum[r] if accum is not None else None for r in range(lres)]
+    idxv, cntv, outv, scv = list(idx), list(count), list(out), list(scores)
+    lens_d, kk_d = lk_d[0], lk_d[1]
+    fork, join = torch.cuda.Event(), torch.cuda.Event()
+    sel = [torch.cuda.Event() for _ in range(L)]
 
     def one(t):
         q_all[t].copy_(q_h[t], non_blocking=True)
@@ -519,38 +563,69 @@ def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all,
             for b in range(B):
                 Kall[:, b, :, pos[t][b]].copy_(stage_k[:, b])
                 Vall[:, b, :, pos[t][b]].copy_(stage_v[:, b])
+        if not args.serial:
+            fork.record(stream)
+            side.wait_event(fork)
         for l in range(L):
             r = l % lres
-            hill.hill_evict_step(desc, q_all[t, l], Kall[r], Vall[r], lk_d[0], lk_d[1], w.max_k, mode,
-                                 accum[r] if accum is not None else None, scores[l], idx[l], count[l], out[l],
-                                 ws, stream)
+            hill.hill_evict_step(desc, qv[t][l], Kv[r], Vv[r], lens_d, kk_d, w.max_k, mode, accv[r], scv[l],
+                                 idxv[l], cntv[l], outv[l] if args.serial else None, ws, stream)
+            if not args.serial:
+                sel[l].record(stream)
+                side.wait_event(sel[l])
+                hill.hill_gather_sparse_attn(desc, qv[t][l], Kv[r], Vv[r], idxv[l], cntv[l], w.max_k, outv[l],
+                                             ws_attn, side)
+        if not args.serial:
+            join.record(side)
+            stream.wait_event(join)
         idx_h.copy_(idx, non_blocking=True)
         cnt_h.copy_(count, non_blocking=True)
         out_h.copy_(out, non_blocking=True)
 
-    with torch.cuda.stream(stream):
-        for i in range(args.warmup):
-            one(i % S)
-    stream.synchronize()
-    barrier(dev)
-    torch.cuda.synchronize(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for t in order:
+    def timed(step_fn):
+        with torch.cuda.stream(stream):
+            for i in range(args.warmup):
+                step_fn(i % S)
+        stream.synchronize()
+        barrier(dev)
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for t in order:
+                step_fn(t)
+            e1.record(stream)
+        stream.synchronize()
+        barrier(dev)
+        hill.hill_sync_status(stream)
+        return max_over_ranks(e0.elapsed_time(e1), dev)
+
+    # eager: every call issued from Python at every step
+    ms_eager = timed(one)
+    # the same calls and copies captured once per decode step and replayed: the
+    # graph of step t copies that step's inputs in from pinned host memory and
+    # its results out to pinned host memory at every replay
+    graphs = []
+    for t in range(S):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
             one(t)
-        e1.record(stream)
-    stream.synchronize()
-    barrier(dev)
-    hill.hill_sync_status(stream)
-    ms = max_over_ranks(e0.elapsed_time(e1), dev)
+        graphs.append(g)
+    ms = timed(lambda t: graphs[t].replay())
+    del graphs
     tokens = sum(L * sum(w.lens_at(t)) for t in order)
     h2d = (q_h[0].numel() * q_h.element_size() + 2 * newk_h[0].numel() * newk_h.element_size()
            + lk_h[0].numel() * 4)
     d2h = idx_h.numel() * 4 + cnt_h.numel() * 4 + out_h.numel() * 4
+    calls = ("hill_evict_step per layer" if args.serial else
+             "hill_evict_step (no attention) + hill_gather_sparse_attn on a second stream, per layer")
     return {"value": round(world * tokens / (ms / 1e3), 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": round(ms / len(order), 4),
-            "api": "hill_evict_step per layer, eager (no graph)"}
+            "api": calls + ", with the step's host-to-device input copies and device-to-host result copies, "
+                           "captured per decode step in a CUDA graph and replayed",
+            "eager": {"value": round(world * tokens / (ms_eager / 1e3), 1),
+                      "ms_per_step": round(ms_eager / len(order), 4),
+                      "api": calls + ", issued from Python at every step (no graph)"}}
 
 
 def cpu_baseline(w, lres, Kall, Vall, q_all, mode, seconds=10.0):
@@ -637,9 +712,9 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--overlap", action="store_true",
-                    help="layer-pipelined schedule: attention of layer l on a second stream, overlapping the "
-                         "evaluation of layer l+1")
+    ap.add_argument("--serial", action="store_true",
+                    help="time the serial schedule (one fused hill_evict_step per layer) as the headline; the "
+                         "default is the layer-pipelined schedule of Sec. 4.3 (both are measured and reported)")
     ap.add_argument("--f8", action="store_true",
                     help="asymmetric-precision scoring (Sec. 4.4) from an E4M3 key shadow (hill_evict_step_f8)")
     ap.add_argument("--bkp-recent", type=int, default=-1,
