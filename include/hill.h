@@ -18,6 +18,14 @@
  * - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
  *   stream).  A returned HILL_OK means the work was enqueued.  Two calls that
  *   share a workspace must be ordered on the GPU (same stream).
+ * - Kernels are launched as programmatic dependents of the previous kernel on
+ *   the stream.  The first kernel of a call may read the call's inputs (q,
+ *   the 16-bit K cache, lens, k) before its dependency wait, so those must be
+ *   complete when the call is issued in stream order: work that writes them
+ *   must not be a kernel that triggers its dependents early
+ *   (griddepcontrol.launch_dependents) and writes them afterwards.  Ordinary
+ *   kernels and copies satisfy this.  Outputs and workspace are written only
+ *   after the wait.
  * - Host-side validation failures return immediately and launch nothing.
  *   Launch failures return HILL_ERR_CUDA.  Conditions only visible on the
  *   device (a budget larger than max_k, a selected index outside the cache, a

@@ -150,6 +150,13 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const void* tmap, int 
       : "memory");
 }
 
+// Bring a 4-D box of a tensor map into L2 (no shared memory, no barrier).
+__device__ __forceinline__ void tma_prefetch_l2_4d(const void* tmap, int c0, int c1, int c2, int c3) {
+  asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(tmap), "r"(c0),
+               "r"(c1), "r"(c2), "r"(c3)
+               : "memory");
+}
+
 // 2^x on the special-function unit (ex2.approx.ftz.f32, relative error about
 // 2^-22; 2^-inf = +0).  Softmax weights are formed as 2^(z*log2(e) - m) with
 // the logits kept pre-scaled by log2(e), which equals e^(z - m').

@@ -60,6 +60,8 @@ struct ScoreCfg {
   static constexpr int kBytes = kOffFlag + 16 + 1024;        // + alignment slack
 };
 
+constexpr int kL2Ahead = 4;   // stages per warp brought into L2 before the dependency wait
+
 __device__ __forceinline__ int find_seq(const int* tstart, int B, int item) {
   int lo = 0, hi = B;  // tstart[lo] <= item < tstart[hi]
   while (hi - lo > 1) {
@@ -108,14 +110,14 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
     *abort_flag = 0;
     prefetch_tmap(&a.kmap);
   }
-  pdl_wait();
-  pdl_launch_dependents();
-  if (a.hist0) {   // this CTA's share of the leading-digit histogram, zeroed for the normalisation
-    const int64_t per = (a.hist0_words + gridDim.x - 1) / gridDim.x;
-    const int64_t w0 = min((int64_t)blockIdx.x * per, a.hist0_words);
-    const int64_t w1 = min(w0 + per, a.hist0_words);
-    for (int64_t w = w0 + threadIdx.x; w < w1; w += kThreads) a.hist0[w] = 0u;
-  }
+  // Before the dependency wait this kernel reads only the inputs of the call
+  // (lengths, and with 16-bit keys the K cache itself), which the caller has
+  // completed before the call (include/hill.h): it builds the tile table and
+  // starts the first stages of every warp, so their DRAM latency overlaps the
+  // end of the previous kernel.  Every write to global memory (the histogram
+  // zeroing, logits, partials, scores) comes after the wait.  The E4M3 shadow
+  // is written by hill_quantize_k, possibly the kernel just before, so with
+  // F8 the first loads wait too.
   for (int b = threadIdx.x; b < B; b += kThreads) {
     int len = a.lens[b];
     if (len < 0 || len > cap) {
@@ -138,14 +140,13 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   const int n_items = tstart[B];
   const int per = (n_items + gridDim.x - 1) / gridDim.x;     // items per CTA
   const int it_lo = min(n_items, (int)blockIdx.x * per), it_hi = min(n_items, it_lo + per);
-  if (it_lo >= it_hi) return;
   const int ng = (Hkv - warp + kNW - 1) / kNW;   // KV heads of this warp per tile (0 .. kMaxNg)
 
   const uint64_t pol = l2_evict_first_policy();
   const uint32_t stage0 = base_addr + warp * kSW * kSlotBytes;
   const uint32_t bar0 = base_addr + Cfg::kOffBar + warp * kSW * 8;
   const uint32_t scale0 = base_addr + Cfg::kOffScale + warp * kSW * kT * 4;   // F8 only
-  const int b_first = find_seq(tstart, B, it_lo);
+  const int b_first = it_lo < it_hi ? find_seq(tstart, B, it_lo) : 0;
 
   auto advance = [&](Cursor& c) {
     if (++c.r >= ng) {
@@ -179,13 +180,43 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   // prologue: the first kSW stages of this warp
   Cursor pc{it_lo, 0, b_first};
   uint32_t issued = 0, is_slot = 0;
-  if (ng > 0) {
-    for (; issued < (uint32_t)kSW && pc.item < it_hi; ++issued) {
-      if (lane == 0) issue(pc, is_slot);
-      is_slot = is_slot + 1 == (uint32_t)kSW ? 0u : is_slot + 1;
-      advance(pc);
+  auto prologue = [&]() {
+    if (ng > 0) {
+      for (; issued < (uint32_t)kSW && pc.item < it_hi; ++issued) {
+        if (lane == 0) issue(pc, is_slot);
+        is_slot = is_slot + 1 == (uint32_t)kSW ? 0u : is_slot + 1;
+        advance(pc);
+      }
+    }
+  };
+  if constexpr (!F8) {
+    prologue();
+    // and the next kL2Ahead stages into L2, so that the HBM stream keeps going
+    // while the previous kernel finishes
+    if (lane == 0 && ng > 0) {
+      Cursor lc = pc;
+      for (int u = 0; u < kL2Ahead && lc.item < it_hi; ++u) {
+        const int j0 = (lc.item - tstart[lc.b]) * kT;
+        const int g = warp + lc.r * kNW;
+        const int c1 = a.kdim_tok == 1 ? j0 : (a.kdim_head == 1 ? g : lc.b);
+        const int c2 = a.kdim_tok == 2 ? j0 : (a.kdim_head == 2 ? g : lc.b);
+        const int c3 = a.kdim_tok == 3 ? j0 : (a.kdim_head == 3 ? g : lc.b);
+        tma_prefetch_l2_4d(&a.kmap, 0, c1, c2, c3);
+        tma_prefetch_l2_4d(&a.kmap, 64, c1, c2, c3);
+        advance(lc);
+      }
     }
   }
+  pdl_wait();
+  pdl_launch_dependents();
+  if (a.hist0) {   // this CTA's share of the leading-digit histogram, zeroed for the normalisation
+    const int64_t hper = (a.hist0_words + gridDim.x - 1) / gridDim.x;
+    const int64_t w0 = min((int64_t)blockIdx.x * hper, a.hist0_words);
+    const int64_t w1 = min(w0 + hper, a.hist0_words);
+    for (int64_t w = w0 + threadIdx.x; w < w1; w += kThreads) a.hist0[w] = 0u;
+  }
+  if (it_lo >= it_hi) return;
+  if constexpr (F8) prologue();
 
   // fragment coordinates (mma.sync m16n8k16): C row = token lane/4 (+8),
   // C columns = heads 2*(lane%4) and 2*(lane%4)+1 of the group
