@@ -78,3 +78,58 @@ def test_pipelined_layers_equal_serial(H):
         for got in ((idx1, cnt1, out1), (idx2, cnt2, out2)):
             assert torch.equal(got[0][l], idx0[l]) and torch.equal(got[1][l], cnt0[l])
             assert torch.equal(got[2][l], out0[l])
+
+
+@pytest.mark.parametrize("wl", [2, 4])
+def test_pipelined_full_size_equals_serial(H, wl):
+    """The benchmark's default schedule at full per-layer size (4K MHA and
+    128K GQA workloads, three layers, last decode step, in a CUDA graph as
+    the benchmark runs it) gives the serial step's selection and attention
+    bit for bit; the serial step itself is checked against the oracle by the
+    sampled full-size parity tests."""
+    w = inputs.config(wl)
+    L = 3
+    t = w.steps - 1
+    cache = [inputs.layer_cache(w, l, device="cuda") for l in range(L)]
+    qs = [inputs.step_query(w, l, t, device="cuda") for l in range(L)]
+    lens_t = torch.tensor(w.lens_at(t), dtype=torch.int32, device="cuda")
+    k_t = torch.tensor(w.budget_at(t), dtype=torch.int32, device="cuda")
+    desc = H.make_desc(qs[0], cache[0][0], cache[0][1])
+    ws = [H.alloc_workspace(desc, 0, w.max_k) for _ in range(2)]
+    B, Hq = qs[0].shape[0], qs[0].shape[1]
+
+    def buffers():
+        return ([torch.empty(B, w.max_k, dtype=torch.int32, device="cuda") for _ in range(L)],
+                [torch.empty(B, dtype=torch.int32, device="cuda") for _ in range(L)],
+                [torch.empty(B, Hq, 128, device="cuda") for _ in range(L)])
+
+    idx0, cnt0, out0 = buffers()
+    for l in range(L):
+        H.hill_evict_step(desc, qs[l], cache[l][0], cache[l][1], lens_t, k_t, w.max_k, 0, None, None, idx0[l],
+                          cnt0[l], out0[l], ws[0])
+    H.hill_sync_status()
+    main, side = torch.cuda.Stream(), torch.cuda.Stream()
+    idx1, cnt1, out1 = buffers()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=main):
+        fork = torch.cuda.Event()
+        fork.record(main)
+        side.wait_event(fork)
+        for l in range(L):
+            H.hill_evict_step(desc, qs[l], cache[l][0], cache[l][1], lens_t, k_t, w.max_k, 0, None, None,
+                              idx1[l], cnt1[l], None, ws[0], main)
+            sel = torch.cuda.Event()
+            sel.record(main)
+            side.wait_event(sel)
+            H.hill_gather_sparse_attn(desc, qs[l], cache[l][0], cache[l][1], idx1[l], cnt1[l], w.max_k, out1[l],
+                                      ws[1], side)
+        join = torch.cuda.Event()
+        join.record(side)
+        main.wait_event(join)
+    for _ in range(2):
+        g.replay()
+    torch.cuda.synchronize()
+    H.hill_sync_status()
+    for l in range(L):
+        assert torch.equal(idx1[l], idx0[l]) and torch.equal(cnt1[l], cnt0[l])
+        assert torch.equal(out1[l], out0[l])
