@@ -239,7 +239,7 @@ const char* hill_status_string(hill_status status);
  *    before any stream capture.
  *  - A call needing more scratch than the array holds returns
  *    HILL_ERR_WORKSPACE without launching anything.  ATTN mode needs about
- *    4*B*cap*(H + 1) + 8*B*H*SMs bytes; RAW about 4*B*cap.
+ *    4*B*cap*(H + 1) + 8*B*H*(SMs + 1) bytes; RAW about 4*B*cap.
  *  - All calls share the array, and it keeps whatever the last call left;
  *    no entry of it needs to start at zero (a call reads only what it wrote).
  *    Calls that overlap on the GPU (two streams, or two host threads without

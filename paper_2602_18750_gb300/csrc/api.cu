@@ -158,7 +158,7 @@ hill_status check_desc(const hill_desc* d) {
 }
 
 struct Layout {
-  size_t scores, logits, partials, hist0, attn_part, total;
+  size_t scores, logits, partials, stats, hist0, attn_part, total;
   bool has_hist0;
   int score_grid, attn_grid, splits;
 };
@@ -184,6 +184,9 @@ Layout layout_for(const hill_desc* d, int mode, int max_k, int sms) {
   if (mode == HILL_SCORE_ATTN) off += align_up(B * H * cap * sizeof(float));
   L.partials = off;
   if (mode == HILL_SCORE_ATTN) off += align_up(B * (size_t)L.score_grid * H * sizeof(float2));
+  // combined (max, 1/sum) per (b, h), when the normalisation runs in two kernels
+  L.stats = off;
+  if (mode == HILL_SCORE_ATTN) off += align_up(B * H * sizeof(float2));
   // leading-digit histogram of the selection key, built by the ATTN
   // normalisation when a selection follows (max_k > 0)
   L.hist0 = off;
@@ -256,7 +259,10 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   f.recent = recent;
   f.kvh = kvh ? 1 : 0;
   f.Hkv = d->num_kv_heads;
-  return from_cuda(counted(launch_attn_finalize(f, st), 1));
+  f.stats = reinterpret_cast<float2*>(base + L.stats);
+  int kernels = 0;
+  const cudaError_t e = launch_attn_finalize(f, di.sms, st, &kernels);
+  return from_cuda(counted(e, kernels));
 }
 
 hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens, const int32_t* k,

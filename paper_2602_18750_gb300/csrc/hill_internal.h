@@ -44,6 +44,7 @@ struct FinalizeArgs {
   int recent;         // tokens j >= len - min(recent, len) are left out of hist0 (pinned, not ranked)
   int kvh;            // 1: scores/accum are [B][Hkv][cap], the sum over each KV head's G query heads
   int Hkv;
+  float2* stats;      // [B][H] (max, 1/sum) per head, or NULL: every finalize CTA combines the partials
 };
 
 struct QuantArgs {
@@ -139,7 +140,8 @@ int score_warps();
 int score_max_batch();
 int score_max_kv_heads(int G);
 cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8, int grid, cudaStream_t st);
-cudaError_t launch_attn_finalize(const FinalizeArgs& a, cudaStream_t st);
+// Launches the normalisation (one or two kernels: *kernels is set to the count).
+cudaError_t launch_attn_finalize(const FinalizeArgs& a, int sms, cudaStream_t st, int* kernels);
 
 // selftest.cu
 cudaError_t launch_selftest_wait(unsigned long long limit_ns, unsigned* err, cudaStream_t st);

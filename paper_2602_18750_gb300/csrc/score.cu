@@ -488,6 +488,9 @@ constexpr int kFinPartMax = 32;                    // partials per thread held i
 constexpr int kHistBins = 2048;                    // leading 11 bits of the order-preserving key
 constexpr int kFinZReg = 32;                       // logits per token held in registers
 
+// STATS: the per-head (max, 1/sum) come from hill_attn_stats_kernel instead of
+// every CTA combining the partials itself (long sequences: many CTAs).
+template <bool STATS>
 __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(FinalizeArgs a) {
   extern __shared__ float fsm[];
   float* mh = fsm;            // [H]
@@ -535,9 +538,16 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   float zr[kFinZReg];
 #pragma unroll
   for (int u = 0; u < kFinZReg; ++u) zr[u] = (valid && u < a.H) ? zp[(int64_t)u * a.cap] : 0.f;
+  if constexpr (STATS) {
+    for (int h = threadIdx.x; h < a.H; h += kFinThreads) {
+      const float2 st = a.stats[(int64_t)b * a.H + h];
+      mh[h] = st.x;
+      il[h] = st.y;
+    }
+  }
   const float2* pb = a.partials + (int64_t)b * a.nslot * a.H;
   const int sub = threadIdx.x % kFinPartThreads;
-  for (int h = threadIdx.x / kFinPartThreads; h < a.H; h += kFinThreads / kFinPartThreads) {
+  for (int h = threadIdx.x / kFinPartThreads; !STATS && h < a.H; h += kFinThreads / kFinPartThreads) {
     float2 p[kFinPartMax];
 #pragma unroll
     for (int u = 0; u < kFinPartMax; ++u) {
@@ -636,6 +646,68 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   }
 }
 
+// Combine the per-CTA (max, sum) partials of one (b, h) into its softmax
+// statistics (max, 1 / sum) in the base-2 scale: one warp per pair, each lane
+// taking every 32nd partial with a running maximum, the lanes then merged by
+// shuffles.  Used ahead of hill_attn_finalize_kernel<true> when the
+// normalisation has many CTAs per sequence.
+constexpr int kStatsWarps = 8;
+constexpr int kStatsPer = 8;   // partials per lane whose loads are in flight together
+
+__global__ void __launch_bounds__(kStatsWarps * 32) hill_attn_stats_kernel(FinalizeArgs a) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int pair = blockIdx.x * kStatsWarps + warp;
+  if (pair >= a.B * a.H) return;
+  const int b = pair / a.H, h = pair - b * a.H;
+  // the slots 0 .. ns-1 of b (lengths are inputs of the call: read before the wait)
+  int f = 0, t = 0;
+  for (int bb = lane; bb < a.B; bb += 32) {
+    int lb = a.lens[bb];
+    lb = lb < 0 ? 0 : (lb > a.cap ? a.cap : lb);
+    const int tiles = (lb + kT - 1) / kT;
+    f += bb < b ? tiles : 0;
+    t += tiles;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    f += __shfl_xor_sync(0xffffffffu, f, o);
+    t += __shfl_xor_sync(0xffffffffu, t, o);
+  }
+  int len = a.lens[b];
+  len = len < 0 ? 0 : (len > a.cap ? a.cap : len);
+  const int items = (len + kT - 1) / kT;
+  const int per = (t + a.nslot - 1) / a.nslot;
+  const int ns = items == 0 ? 0 : (f + items - 1) / per - f / per + 1;
+  pdl_wait();
+  pdl_launch_dependents();
+  const float2* pb = a.partials + (int64_t)b * a.nslot * a.H + h;
+  float m = -INFINITY, l = 0.f;
+  for (int s0 = lane; s0 < ns; s0 += 32 * kStatsPer) {
+    float2 p[kStatsPer];
+#pragma unroll
+    for (int u = 0; u < kStatsPer; ++u) {
+      const int s = s0 + 32 * u;
+      p[u] = s < ns ? pb[(int64_t)s * a.H] : make_float2(-INFINITY, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < kStatsPer; ++u) {
+      if (!(p[u].y > 0.f)) continue;
+      const float mn = fmaxf(m, p[u].x);
+      l = l * ex2(m - mn) + p[u].y * ex2(p[u].x - mn);
+      m = mn;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float mo = __shfl_xor_sync(0xffffffffu, m, o);
+    const float lo = __shfl_xor_sync(0xffffffffu, l, o);
+    const float mn = fmaxf(m, mo);
+    l = (l > 0.f ? l * ex2(m - mn) : 0.f) + (lo > 0.f ? lo * ex2(mo - mn) : 0.f);
+    m = mn;
+  }
+  if (lane == 0) a.stats[pair] = make_float2(m, 1.f / l);
+}
+
 template <int DT, int G, bool RAW, bool F8>
 cudaError_t launch_score_t(const ScoreArgs& a, int grid, cudaStream_t st) {
   const size_t smem = (size_t)ScoreCfg<G, F8>::kBytes;
@@ -686,10 +758,21 @@ cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8
   return f8 ? launch_score_m<1, true>(a, G, raw, grid, st) : launch_score_m<1, false>(a, G, raw, grid, st);
 }
 
-cudaError_t launch_attn_finalize(const FinalizeArgs& a, cudaStream_t st) {
+cudaError_t launch_attn_finalize(const FinalizeArgs& a, int sms, cudaStream_t st, int* kernels) {
   dim3 grid((a.cap + kFinChunk - 1) / kFinChunk, a.B);
   const size_t smem = 2 * a.H * sizeof(float) + (a.hist0 ? kHistBins * sizeof(uint32_t) : 0);
-  return launch_pdl(hill_attn_finalize_kernel, grid, dim3(kFinThreads), smem, st, 0, a);
+  // more than two normalisation CTAs per SM: combine the partials once per
+  // (b, h) in a kernel of their own instead of once per CTA
+  if (a.stats && (long long)grid.x * grid.y > 2LL * sms) {
+    *kernels = 2;
+    const int pairs = a.B * a.H;
+    cudaError_t e = launch_pdl(hill_attn_stats_kernel, dim3((pairs + kStatsWarps - 1) / kStatsWarps),
+                               dim3(kStatsWarps * 32), 0, st, 0, a);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(hill_attn_finalize_kernel<true>, grid, dim3(kFinThreads), smem, st, 0, a);
+  }
+  *kernels = 1;
+  return launch_pdl(hill_attn_finalize_kernel<false>, grid, dim3(kFinThreads), smem, st, 0, a);
 }
 
 }  // namespace hill
