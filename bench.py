@@ -211,7 +211,7 @@ def describe(w, lres, mode_name):
         "budget": (f"floor({w.budget_frac}*len)" if w.budget_tokens is None else w.budget_tokens),
         "kv_dtype": str(w.dtype).replace("torch.", ""), "skew": w.kind, "importance": mode_name,
         "accumulate": w.accumulate,
-        "l2": "inputs larger than L2 (each layer's K > 129 MB; layers distinct), no flush",
+        "l2": "inputs larger than L2 (each layer's K > 129 MB; consecutive layers distinct), no flush",
     }
 
 
@@ -232,6 +232,13 @@ def run_ours(args):
 
     mode = hill.HILL_SCORE_ATTN if args.mode == "attn" else hill.HILL_SCORE_RAW
     w, lres = workload_for(args.workload, replica_seed(args.seed, rank), args.layers_resident)
+    if args.layers_resident is None:
+        # keep as many layers resident as fit in 70 % of the free device memory
+        # (the 64K sweep point needs 8.6 GB of K/V per layer); layers beyond
+        # that reuse the resident ones cyclically, each larger than L2
+        per_layer = 2 * w.batch * w.kv_heads * w.capacity * w.head_dim * torch.finfo(w.dtype).bits // 8
+        free = torch.cuda.mem_get_info(dev)[0]
+        lres = max(1, min(lres, int(0.7 * free) // per_layer))
     L, S, B, Hq, Hkv, d = w.layers, w.steps, w.batch, w.heads, w.kv_heads, w.head_dim
     cap, max_k = w.capacity, w.max_k
     bkp = args.bkp_recent >= 0
