@@ -4,13 +4,16 @@
 // Gather + split-K flash decode on persistent CTAs.  The work is a list of
 // batches: (sequence b, KV head g, batch bi of 32 consecutive entries of
 // b's index list), ordered b, g, bi.  Every warp of the grid owns one
-// contiguous segment of that list and streams it through two shared-memory
-// slots.  A batch's 32 K rows and 32 V rows (tokens idx[b][32*bi + i]) are
-// gathered with 16-byte asynchronous copies (one cp.async group per batch, a
-// half-warp per 256-byte row) into an XOR-swizzled layout that ldmatrix reads
-// without bank conflicts; rows of absent tokens are zero-filled by the copies
-// themselves.  The index entries of the batch after next are loaded while the
-// current one computes and are checked only when that batch is issued.  (TMA
+// contiguous segment of that list and streams it through a K region and a V
+// region of shared memory.  A batch's 32 K rows and 32 V rows (tokens
+// idx[b][32*bi + i]) are gathered with 16-byte asynchronous copies (a
+// half-warp per 256-byte row; the K rows and the V rows are separate copy
+// groups, so K of the next batch is in flight while this batch's softmax and
+// P.V run, and V of the next batch while the next S runs) into an
+// XOR-swizzled layout that ldmatrix reads without bank conflicts; rows of
+// absent tokens are zero-filled by the copies themselves.  The index entries
+// of the batch after next are loaded with the K copies and are checked only
+// when that batch is issued.  (TMA
 // alternatives were measured slower on the same layout: 256-byte bulk copies
 // per row are bound by the copy engine's request rate, and tile::gather4 loads
 // reached about 85 % of the cp.async throughput; neither depends on how

@@ -26,10 +26,15 @@
 //         own tokens per head in registers, and the lanes of a head are
 //         combined once, when the CTA leaves a sequence, into one partial per
 //         (sequence, head, CTA).  hill_attn_finalize_kernel combines the
-//         partials and forms s[b,j] = sum_h exp(z[b,h,j] - m_bh) / L_bh.
+//         partials and forms s[b,j] = sum_h exp(z[b,h,j] - m_bh) / L_bh; when
+//         that kernel would need more than two CTAs per SM (long sequences),
+//         hill_attn_stats_kernel first combines the partials once per
+//         (sequence, head).
 //
 // The query rows of a warp's heads are held as mma B fragments in registers
-// for the whole sequence.
+// for the whole sequence.  Before its dependency wait the kernel builds its
+// tile table from the lengths and, with 16-bit keys, starts its first stages
+// (inputs of the call only; every global write comes after the wait).
 #include "hill_internal.h"
 
 namespace hill {
