@@ -99,15 +99,16 @@ def test_bkp_zero_window_equals_plain_select(H):
 
 
 @pytest.mark.parametrize("mode", [ATTN, RAW])
-def test_evict_step_bkp(H, oracle_mod, mode):
+@pytest.mark.parametrize("cap", [1500, 40000], ids=["single-kernel", "statistics-kernel"])
+def test_evict_step_bkp(H, oracle_mod, mode, cap):
     """The fused step with BKP equals hill_score + hill_topk_select_bkp (the
     ATTN path starts its selection from a histogram that must leave the
     pinned window out), matches the oracle's scores and BKP selection, and
     its attention matches the oracle on the GPU's own index set."""
-    B, Hq, Hkv, cap, recent = 3, 8, 2, 1500, 64
-    lens = [1500, 901, 40]
-    k = [150, 90, 10]
-    max_k = 150 + recent
+    B, Hq, Hkv, recent = 3, 8, 2, 64
+    lens = [cap, cap * 3 // 5 + 1, 40]
+    k = [cap // 10, cap // 17, 10]
+    max_k = k[0] + recent
     q, K, V, lens_t = inputs.random_case(B, Hq, Hkv, 128, cap, lens, dtype=torch.float16, seed=21)
     q, K, V, lens_t = q.cuda(), K.cuda(), V.cuda(), lens_t.cuda()
     desc = H.make_desc(q, K, V)

@@ -93,6 +93,25 @@ def test_kvh_accumulates_over_steps(H, oracle_mod, mode):
                     acc_ref.reshape(B * Hkv, cap), rows_lens, np.repeat(k, Hkv), 80)
 
 
+def test_kvh_long_sequences_statistics_kernel(H, oracle_mod):
+    """Per-KV-head sums on the two-kernel normalisation (sequences long
+    enough for more than two normalisation CTAs per SM)."""
+    B, Hq, Hkv, cap = 2, 16, 4, 40000
+    lens, k = [40000, 31111], [3000, 1000]
+    max_k = 3001
+    q, K, V, lens_t = inputs.random_case(B, Hq, Hkv, 128, cap, lens, dtype=torch.bfloat16, seed=77, kind="zipf")
+    q, K, V, lens_t = q.cuda(), K.cuda(), V.cuda(), lens_t.cuda()
+    scores, idx, cnt, out = _run(H, q, K, V, lens_t, k, max_k, ATTN)
+    z = oracle_mod.logits(q.cpu(), K.cpu(), lens)
+    s_ref = oracle_mod.scores_kvh(ATTN, z, lens, Hkv)
+    rows_lens = np.repeat(lens, Hkv).tolist()
+    check_scores(scores.cpu().numpy().reshape(B * Hkv, cap), s_ref.reshape(B * Hkv, cap), rows_lens)
+    check_selection(idx.cpu().numpy().reshape(B * Hkv, max_k), cnt.cpu().numpy().reshape(-1),
+                    s_ref.reshape(B * Hkv, cap), rows_lens, np.repeat(k, Hkv), max_k)
+    o_ref = oracle_mod.sparse_attn_kvh(q.cpu(), K.cpu(), V.cpu(), idx.cpu().numpy(), cnt.cpu().numpy())
+    check_attn(out.cpu().numpy(), o_ref)
+
+
 def test_kvh_with_one_kv_head_equals_sequence_step(H):
     """Hkv = 1: the per-KV-head step is the per-sequence step."""
     B, Hq, cap = 3, 8, 500

@@ -74,6 +74,29 @@ def test_evict_step_matches_oracle(H, oracle_mod, mode, dtype, shape):
     check_attn(ev.out.cpu().numpy(), out_ref)
 
 
+@pytest.mark.parametrize("dtype", [torch.float16, torch.bfloat16])
+def test_long_sequences_statistics_kernel(H, oracle_mod, dtype):
+    """Sequences long enough that the normalisation takes more than two CTAs
+    per SM (2 x 157 CTAs on 152 SMs), so the per-head statistics come from
+    hill_attn_stats_kernel; accumulation over two steps included."""
+    B, Hq, Hkv, cap = 2, 8, 8, 40000
+    lens, k = [40000, 23457], [4000, 2345]
+    max_k = 4000
+    accum = torch.zeros(B, cap, device="cuda")
+    acc_ref = np.zeros((B, cap))
+    for step in range(2):
+        q, K, V, lens_t = _case(B, Hq, Hkv, cap, lens, dtype, seed=900 + step, kind="zipf")
+        ev = _run_step(H, q, K, V, lens_t, k, max_k, ATTN, accum=accum)
+        ref = oracle_mod.evict_step(ATTN, q, K, V, lens, k, max_k, with_attn=False)
+        check_scores(ev.scores.cpu().numpy(), ref["s"], lens)
+        for b in range(B):
+            acc_ref[b, : lens[b]] += ref["s"][b, : lens[b]]
+    check_scores(accum.cpu().numpy(), acc_ref, lens, what="accum")
+    check_selection(ev.idx.cpu().numpy(), ev.count.cpu().numpy(), acc_ref, lens, k, max_k)
+    out_ref = oracle_mod.sparse_attn(q, K, V, ev.idx.cpu().numpy(), ev.count.cpu().numpy())
+    check_attn(ev.out.cpu().numpy(), out_ref)
+
+
 @pytest.mark.parametrize("mode", [ATTN, RAW])
 def test_separate_calls_equal_fused_step(H, mode):
     q, K, V, lens_t = _case(2, 8, 2, 400, [400, 250], torch.float16, seed=7)
