@@ -341,7 +341,9 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
     for (int r = 0; r < kMaxNg; ++r) {
       if (r >= ng || !ok) break;
       const int g = warp + r * kNW;
-      if (!mbar_wait(bar0 + cs * 8, cph, a.err)) {
+      // every lane waits; the warp goes on only if all of them saw the phase
+      // complete, so it takes the same path and its shuffles stay converged
+      if (!__all_sync(0xffffffffu, mbar_wait(bar0 + cs * 8, cph, a.err))) {
         ok = false;
         *abort_flag = 1;
         break;
@@ -552,32 +554,39 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   }
   const float2* pb = a.partials + (int64_t)b * a.nslot * a.H;
   const int sub = threadIdx.x % kFinPartThreads;
-  for (int h = threadIdx.x / kFinPartThreads; !STATS && h < a.H; h += kFinThreads / kFinPartThreads) {
+  // A warp covers kHeadsPerWarp consecutive heads per pass.  The loop runs
+  // while the warp's first head exists, so every lane of a warp takes the
+  // same trips and the full-mask shuffles below always have all 32 lanes;
+  // lanes whose head is past H combine nothing and write nothing.
+  constexpr int kHeadsPerWarp = 32 / kFinPartThreads;
+  for (int h0 = (threadIdx.x >> 5) * kHeadsPerWarp; !STATS && h0 < a.H; h0 += kFinThreads / kFinPartThreads) {
+    const int h = h0 + (threadIdx.x & 31) / kFinPartThreads;
+    const bool hv = h < a.H;
     float2 p[kFinPartMax];
 #pragma unroll
     for (int u = 0; u < kFinPartMax; ++u) {
       const int s = sub + u * kFinPartThreads;
-      p[u] = s < ns ? pb[(int64_t)s * a.H + h] : make_float2(-INFINITY, 0.f);
+      p[u] = hv && s < ns ? pb[(int64_t)s * a.H + h] : make_float2(-INFINITY, 0.f);
     }
     float m = -INFINITY;
 #pragma unroll
     for (int u = 0; u < kFinPartMax; ++u) m = fmaxf(m, p[u].x);
-    // slots beyond kFinPartMax * kFinPartThreads (grids of more than 256
-    // CTAs) are folded in sequentially
-    for (int s = sub + kFinPartMax * kFinPartThreads; s < ns; s += kFinPartThreads)
+    // slots beyond kFinPartMax * kFinPartThreads (more than 256 scoring
+    // CTAs on one sequence) are folded in sequentially
+    for (int s = sub + kFinPartMax * kFinPartThreads; hv && s < ns; s += kFinPartThreads)
       m = fmaxf(m, pb[(int64_t)s * a.H + h].x);
 #pragma unroll
     for (int o = kFinPartThreads / 2; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
     float l = 0.f;
 #pragma unroll
     for (int u = 0; u < kFinPartMax; ++u) l += p[u].y > 0.f ? p[u].y * ex2(p[u].x - m) : 0.f;
-    for (int s = sub + kFinPartMax * kFinPartThreads; s < ns; s += kFinPartThreads) {
+    for (int s = sub + kFinPartMax * kFinPartThreads; hv && s < ns; s += kFinPartThreads) {
       const float2 q = pb[(int64_t)s * a.H + h];
       l += q.y > 0.f ? q.y * ex2(q.x - m) : 0.f;
     }
 #pragma unroll
     for (int o = kFinPartThreads / 2; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-    if (sub == 0) {
+    if (sub == 0 && hv) {
       mh[h] = m;
       il[h] = 1.f / l;
     }

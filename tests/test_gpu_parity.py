@@ -51,6 +51,9 @@ SHAPES = [
     (2, 32, 8, 700, [700, 1], [64, 5]),
     (2, 8, 1, 300, [300, 299], [30, 299]),
     (4, 4, 2, 129, [129, 0, 64, 95], [13, 3, 64, 0]),
+    # fewer query heads than one warp of the normalisation combines
+    (2, 2, 1, 300, [300, 150], [30, 15]),
+    (2, 1, 1, 257, [257, 100], [20, 100]),
 ]
 
 
