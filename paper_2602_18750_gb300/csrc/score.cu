@@ -492,8 +492,54 @@ constexpr int kFinThreads = 256;
 constexpr int kFinChunk = kFinThreads;
 constexpr int kFinPartThreads = 8;                 // threads combining one head
 constexpr int kFinPartMax = 32;                    // partials per thread held in registers
+constexpr int kFinPartFew = 4;                     // the same when a sequence has few (<= 32) slots
 constexpr int kHistBins = 2048;                    // leading 11 bits of the order-preserving key
 constexpr int kFinZReg = 32;                       // logits per token held in registers
+
+// Combine the ns per-CTA partials (max, sum) of every head of sequence b into
+// mh[h] (max) and il[h] (1 / sum): kFinPartThreads threads per head, each
+// holding PM partials in registers with all their loads in flight; slots
+// beyond PM * kFinPartThreads are folded in sequentially.  A warp covers
+// kHeadsPerWarp consecutive heads per pass.  The loop runs while the warp's
+// first head exists, so every lane of a warp takes the same trips and the
+// full-mask shuffles always have all 32 lanes; lanes whose head is past H
+// combine nothing and write nothing.
+template <int PM>
+__device__ __forceinline__ void combine_partials(const FinalizeArgs& a, int b, int ns, float* mh, float* il) {
+  const float2* pb = a.partials + (int64_t)b * a.nslot * a.H;
+  const int sub = threadIdx.x % kFinPartThreads;
+  constexpr int kHeadsPerWarp = 32 / kFinPartThreads;
+  for (int h0 = (threadIdx.x >> 5) * kHeadsPerWarp; h0 < a.H; h0 += kFinThreads / kFinPartThreads) {
+    const int h = h0 + (threadIdx.x & 31) / kFinPartThreads;
+    const bool hv = h < a.H;
+    float2 p[PM];
+#pragma unroll
+    for (int u = 0; u < PM; ++u) {
+      const int s = sub + u * kFinPartThreads;
+      p[u] = hv && s < ns ? pb[(int64_t)s * a.H + h] : make_float2(-INFINITY, 0.f);
+    }
+    float m = -INFINITY;
+#pragma unroll
+    for (int u = 0; u < PM; ++u) m = fmaxf(m, p[u].x);
+    for (int s = sub + PM * kFinPartThreads; hv && s < ns; s += kFinPartThreads)
+      m = fmaxf(m, pb[(int64_t)s * a.H + h].x);
+#pragma unroll
+    for (int o = kFinPartThreads / 2; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    float l = 0.f;
+#pragma unroll
+    for (int u = 0; u < PM; ++u) l += p[u].y > 0.f ? p[u].y * ex2(p[u].x - m) : 0.f;
+    for (int s = sub + PM * kFinPartThreads; hv && s < ns; s += kFinPartThreads) {
+      const float2 q = pb[(int64_t)s * a.H + h];
+      l += q.y > 0.f ? q.y * ex2(q.x - m) : 0.f;
+    }
+#pragma unroll
+    for (int o = kFinPartThreads / 2; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+    if (sub == 0 && hv) {
+      mh[h] = m;
+      il[h] = 1.f / l;
+    }
+  }
+}
 
 // STATS: the per-head (max, 1/sum) come from hill_attn_stats_kernel instead of
 // every CTA combining the partials itself (long sequences: many CTAs).
@@ -552,44 +598,10 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
       il[h] = st.y;
     }
   }
-  const float2* pb = a.partials + (int64_t)b * a.nslot * a.H;
-  const int sub = threadIdx.x % kFinPartThreads;
-  // A warp covers kHeadsPerWarp consecutive heads per pass.  The loop runs
-  // while the warp's first head exists, so every lane of a warp takes the
-  // same trips and the full-mask shuffles below always have all 32 lanes;
-  // lanes whose head is past H combine nothing and write nothing.
-  constexpr int kHeadsPerWarp = 32 / kFinPartThreads;
-  for (int h0 = (threadIdx.x >> 5) * kHeadsPerWarp; !STATS && h0 < a.H; h0 += kFinThreads / kFinPartThreads) {
-    const int h = h0 + (threadIdx.x & 31) / kFinPartThreads;
-    const bool hv = h < a.H;
-    float2 p[kFinPartMax];
-#pragma unroll
-    for (int u = 0; u < kFinPartMax; ++u) {
-      const int s = sub + u * kFinPartThreads;
-      p[u] = hv && s < ns ? pb[(int64_t)s * a.H + h] : make_float2(-INFINITY, 0.f);
-    }
-    float m = -INFINITY;
-#pragma unroll
-    for (int u = 0; u < kFinPartMax; ++u) m = fmaxf(m, p[u].x);
-    // slots beyond kFinPartMax * kFinPartThreads (more than 256 scoring
-    // CTAs on one sequence) are folded in sequentially
-    for (int s = sub + kFinPartMax * kFinPartThreads; hv && s < ns; s += kFinPartThreads)
-      m = fmaxf(m, pb[(int64_t)s * a.H + h].x);
-#pragma unroll
-    for (int o = kFinPartThreads / 2; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-    float l = 0.f;
-#pragma unroll
-    for (int u = 0; u < kFinPartMax; ++u) l += p[u].y > 0.f ? p[u].y * ex2(p[u].x - m) : 0.f;
-    for (int s = sub + kFinPartMax * kFinPartThreads; hv && s < ns; s += kFinPartThreads) {
-      const float2 q = pb[(int64_t)s * a.H + h];
-      l += q.y > 0.f ? q.y * ex2(q.x - m) : 0.f;
-    }
-#pragma unroll
-    for (int o = kFinPartThreads / 2; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-    if (sub == 0 && hv) {
-      mh[h] = m;
-      il[h] = 1.f / l;
-    }
+  if constexpr (!STATS) {
+    // ns is the same for the whole CTA, so every warp takes the same branch
+    if (ns <= kFinPartThreads * kFinPartFew) combine_partials<kFinPartFew>(a, b, ns, mh, il);
+    else combine_partials<kFinPartMax>(a, b, ns, mh, il);
   }
   if (a.hist0)
     for (int i = threadIdx.x; i < kHistBins; i += kFinThreads) hcount[i] = 0u;
