@@ -29,6 +29,8 @@
 // every instruction covers 8 heads x 16 dims.  When a warp's segment holds
 // all batches of a (b, g) it writes the output; otherwise it writes a partial
 // (max, sum, o) that hill_attn_combine_kernel merges.
+#include <type_traits>
+
 #include "hill_internal.h"
 
 namespace hill {
@@ -445,27 +447,33 @@ __global__ void __launch_bounds__(kCombThreads) hill_attn_combine_kernel(AttnArg
   const float* pp = a.part + (int64_t)bh * a.splits * kPS;
   const int nseg = w1 - w0 + 1;
   float M = -INFINITY, L = 0.f, O = 0.f;
-  constexpr int kU = 16;  // partials per group whose loads are issued together
-  for (int s0 = gi; s0 < nseg; s0 += kCombGroups * kU) {
-    float ms[kU], ls[kU], os[kU];
+  // KU partials per group have their loads issued together; a pair with few
+  // partials (nseg is the same for the whole CTA) takes the short variant
+  auto merge = [&](auto ku) {
+    constexpr int KU = decltype(ku)::value;
+    for (int s0 = gi; s0 < nseg; s0 += kCombGroups * KU) {
+      float ms[KU], ls[KU], os[KU];
 #pragma unroll
-    for (int u = 0; u < kU; ++u) {
-      const int s = s0 + u * kCombGroups;
-      const float* q = pp + (int64_t)s * kPS;
-      ms[u] = s < nseg ? q[0] : -INFINITY;
-      ls[u] = s < nseg ? q[1] : 0.f;
-      os[u] = s < nseg ? q[2 + dd] : 0.f;
-    }
+      for (int u = 0; u < KU; ++u) {
+        const int s = s0 + u * kCombGroups;
+        const float* q = pp + (int64_t)s * kPS;
+        ms[u] = s < nseg ? q[0] : -INFINITY;
+        ls[u] = s < nseg ? q[1] : 0.f;
+        os[u] = s < nseg ? q[2 + dd] : 0.f;
+      }
 #pragma unroll
-    for (int u = 0; u < kU; ++u) {
-      if (ms[u] == -INFINITY) continue;   // past the end (every written partial holds a token)
-      const float mn = fmaxf(M, ms[u]);
-      const float c0 = ex2(M - mn), c1 = ex2(ms[u] - mn);   // partial maxima are in the base-2 scale
-      L = L * c0 + ls[u] * c1;
-      O = O * c0 + os[u] * c1;
-      M = mn;
+      for (int u = 0; u < KU; ++u) {
+        if (ms[u] == -INFINITY) continue;   // past the end (every written partial holds a token)
+        const float mn = fmaxf(M, ms[u]);
+        const float c0 = ex2(M - mn), c1 = ex2(ms[u] - mn);   // partial maxima are in the base-2 scale
+        L = L * c0 + ls[u] * c1;
+        O = O * c0 + os[u] * c1;
+        M = mn;
+      }
     }
-  }
+  };
+  if (nseg <= kCombGroups * 2) merge(std::integral_constant<int, 2>{});
+  else merge(std::integral_constant<int, 16>{});
   s_o[gi][dd] = O;
   if (dd == 0) {
     s_m[gi] = M;
