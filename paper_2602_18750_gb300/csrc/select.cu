@@ -13,9 +13,12 @@
 // 32 slice sums and then the bins of the crossing slice.  A pass ends the
 // search early when the crossing bin is taken whole.  The first pass can
 // start from a histogram of the leading digit that the score normalisation
-// already accumulated (SelectArgs::hist0).  This is the GPU form of the
+// already accumulated (SelectArgs::hist0).  With 8-CTA clusters the keys of
+// the first pass's crossing bucket, when few, are gathered into every CTA so
+// that the later passes need no exchange.  This is the GPU form of the
 // paper's merge of chunked <position, score> blocks (Sec. 4.2): the chunks
-// stay on chip and only bin counts cross between CTAs.
+// stay on chip and only bin counts (or the few candidate keys) cross between
+// CTAs.  All global reads are issued before the first use of any of them.
 //
 // Ties at the boundary go to the lowest token index: with tau the k-th key
 // and r_eq the number of keys equal to tau that must be taken, a token is
@@ -246,14 +249,14 @@ __global__ void __launch_bounds__(kSelThreads) hill_select_kernel(SelectArgs a) 
     if (!local && pass == 0 && C >= kCandMinCluster && bc[2] <= (uint32_t)kCand) {
       // The keys of the crossing bucket are few (typically 1-4 % of the
       // sequence): every CTA gathers all of them from the cluster once, and
-      // passes 1 and 2 then run on that copy inside each CTA, with no
-      // further histogram exchange.  All CTAs hold the same multiset, so
+      // the two remaining passes then run on that copy inside each CTA, with
+      // no further histogram exchange.  All CTAs hold the same multiset, so
       // they reach the same digits.  (Measured: this pays off against the
-      // exchange of 2 x C histograms at C = 8 and loses at C = 2.)  The buffers: this CTA's own candidates
-      // go to `merged` (free after the search above; peers read it until
-      // the compaction's cluster barrier), the gathered copy to histogram
-      // buffer 0 (peers have finished reading it once they pass the barrier
-      // below).
+      // exchange of 2 x C histograms at C = 8 and loses at C = 2.)  The
+      // buffers: this CTA's own candidates go to `merged` (free after the
+      // search above; peers read it until the compaction's cluster barrier),
+      // the gathered copy to histogram buffer 0 (peers have finished reading
+      // it once they pass the barrier below).
       uint32_t* cand = merged;
       if (tid == 0) s_nc = 0;
       __syncthreads();
