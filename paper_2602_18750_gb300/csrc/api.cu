@@ -148,9 +148,10 @@ hill_status check_desc(const hill_desc* d) {
     return HILL_ERR_INVALID_ARG;
   if (d->head_dim != kHeadDim) return HILL_ERR_UNSUPPORTED;
   const int G = d->num_q_heads / d->num_kv_heads;
-  if (G != 1 && G != 2 && G != 4 && G != 8) return HILL_ERR_UNSUPPORTED;
+  // groups of more than 8 query heads per KV head (MQA-like) run in passes of 8
+  if (G != 1 && G != 2 && G != 4 && G != 8 && G != 16 && G != 32) return HILL_ERR_UNSUPPORTED;
   if (d->batch > score_max_batch() || d->batch > attn_max_batch()) return HILL_ERR_UNSUPPORTED;
-  if (d->num_kv_heads > score_max_kv_heads(G)) return HILL_ERR_UNSUPPORTED;
+  if (d->num_kv_heads > score_max_kv_heads(G > 8 ? 8 : G)) return HILL_ERR_UNSUPPORTED;
   // the selection keeps a sequence's keys on chip across at most 8 CTAs
   if (select_smem_bytes(d->capacity, select_cluster_size(d->capacity)) > 220 * 1024)
     return HILL_ERR_UNSUPPORTED;
@@ -243,7 +244,16 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
     a.hist0 = hist0;
     a.hist0_words = (int64_t)d->batch * select_hist_bins();
   }
-  hill_status s = from_cuda(counted(launch_score(a, d->dtype, G, raw, f8, L.score_grid, st), 1));
+  // a group of G > 8 query heads is scored in G / 8 passes over the same keys,
+  // 8 heads each (RAW passes after the first add their sums)
+  const int GP = G > 8 ? 8 : G;
+  a.Gs = G;
+  hill_status s = HILL_OK;
+  for (int p = 0; p < G / GP && s == HILL_OK; ++p) {
+    a.hoff = p * GP;
+    a.raw_add = p > 0 ? 1 : 0;
+    s = from_cuda(counted(launch_score(a, d->dtype, GP, raw, f8, L.score_grid, st), 1));
+  }
   if (s != HILL_OK || raw) return s;
   FinalizeArgs f{};
   f.logits = a.logits;
@@ -318,7 +328,18 @@ hill_status run_attn(const hill_desc* d, const void* q, const void* k, const voi
   a.splits = L.splits;
   a.kvh = kvh ? 1 : 0;
   a.err = di.err;
-  return from_cuda(counted(launch_sparse_attn(a, d->dtype, d->num_q_heads / d->num_kv_heads, L.attn_grid, st), 2));
+  // G > 8 query heads per KV head: passes of 8 heads over the same selected
+  // rows, then one merge of the split partials over all heads
+  const int G = d->num_q_heads / d->num_kv_heads;
+  const int GP = G > 8 ? 8 : G;
+  a.Gs = G;
+  for (int p = 0; p < G / GP; ++p) {
+    a.hoff = p * GP;
+    const bool last = p == G / GP - 1;
+    hill_status s = from_cuda(counted(launch_sparse_attn(a, d->dtype, GP, L.attn_grid, last, st), last ? 2 : 1));
+    if (s != HILL_OK) return s;
+  }
+  return HILL_OK;
 }
 
 }  // namespace

@@ -222,7 +222,7 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
 #pragma unroll
       for (int e = 0; e < 4; ++e) oacc[db][e] = 0.f;
     const auto* q32 = static_cast<const uint32_t*>(a.q);
-    const int64_t row = head_ok ? ((int64_t)b * a.q_sb + (int64_t)(g * G + grp) * a.q_sh) / 2 : 0;
+    const int64_t row = head_ok ? ((int64_t)b * a.q_sb + (int64_t)(g * a.Gs + a.hoff + grp) * a.q_sh) / 2 : 0;
 #pragma unroll
     for (int kb = 0; kb < 8; ++kb) {
       qa[kb][0] = head_ok ? __ldg(q32 + row + kb * 8 + tig) : 0u;
@@ -245,7 +245,7 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
       const int hl = c ? hB : hA;
       if (hl >= G) continue;
       const float m = c ? mB : mA, l = c ? lB : lA;
-      const int h = cg * G + hl;
+      const int h = cg * a.Gs + a.hoff + hl;
       if (whole) {
         float* op = a.out + ((int64_t)cb * a.H + h) * kHeadDim + grp;
         const float inv = l > 0.f ? 1.f / l : 0.f;
@@ -498,23 +498,23 @@ __global__ void __launch_bounds__(kCombThreads) hill_attn_combine_kernel(AttnArg
 }
 
 template <int DT, int G>
-cudaError_t launch_attn_t(const AttnArgs& a, int grid, cudaStream_t st) {
+cudaError_t launch_attn_t(const AttnArgs& a, int grid, bool combine, cudaStream_t st) {
   static int cache[64] = {0};
   auto kern = hill_sparse_attn_kernel<DT, G>;
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), AttnCfg::kSmem, cache);
   if (e != cudaSuccess) return e;
   e = launch_pdl(kern, dim3(grid), dim3(kAThreads), AttnCfg::kSmem, st, 0, a);
-  if (e != cudaSuccess) return e;
+  if (e != cudaSuccess || !combine) return e;
   return launch_pdl(hill_attn_combine_kernel, dim3(a.B * a.H), dim3(kCombThreads), 0, st, 0, a, grid * kAW);
 }
 
 template <int DT>
-cudaError_t launch_attn_d(const AttnArgs& a, int G, int grid, cudaStream_t st) {
+cudaError_t launch_attn_d(const AttnArgs& a, int G, int grid, bool combine, cudaStream_t st) {
   switch (G) {
-    case 1: return launch_attn_t<DT, 1>(a, grid, st);
-    case 2: return launch_attn_t<DT, 2>(a, grid, st);
-    case 4: return launch_attn_t<DT, 4>(a, grid, st);
-    case 8: return launch_attn_t<DT, 8>(a, grid, st);
+    case 1: return launch_attn_t<DT, 1>(a, grid, combine, st);
+    case 2: return launch_attn_t<DT, 2>(a, grid, combine, st);
+    case 4: return launch_attn_t<DT, 4>(a, grid, combine, st);
+    case 8: return launch_attn_t<DT, 8>(a, grid, combine, st);
   }
   return cudaErrorInvalidValue;
 }
@@ -528,8 +528,8 @@ int attn_max_batch() { return kMaxBatchAttn; }
 // ceil(nb / per) + 1 warp segments, and per >= 1.
 int attn_max_segments(int max_k) { return (max_k + kBatch - 1) / kBatch + 1; }
 
-cudaError_t launch_sparse_attn(const AttnArgs& a, int dtype, int G, int grid, cudaStream_t st) {
-  return dtype == 0 ? launch_attn_d<0>(a, G, grid, st) : launch_attn_d<1>(a, G, grid, st);
+cudaError_t launch_sparse_attn(const AttnArgs& a, int dtype, int G, int grid, bool combine, cudaStream_t st) {
+  return dtype == 0 ? launch_attn_d<0>(a, G, grid, combine, st) : launch_attn_d<1>(a, G, grid, combine, st);
 }
 
 }  // namespace hill

@@ -28,6 +28,12 @@ struct ScoreArgs {
   float2* partials;   // ATTN: [B][nslot][H] (max, sum 2^(z2 - max)), base-2 logits z2 = z * log2 e
   int nslot;          // = grid size of the launch
   int kvh;            // RAW with per-KV-head selection: scores/accum [B][Hkv][cap], summed over each group only
+  // Query heads per KV head in the data (Gs) and the first one this launch
+  // handles (hoff): a launch covers heads g * Gs + hoff + [0, G) of every KV
+  // head g.  Gs = G, hoff = 0 except when a group of more than 8 heads is
+  // scored in passes of 8; then RAW passes after the first add to scores
+  // (raw_add) instead of storing.
+  int Gs, hoff, raw_add;
   uint32_t* hist0;    // optional: zero-filled here (hist0_words words) for the normalisation to count into
   int64_t hist0_words;
   unsigned* err;
@@ -84,6 +90,7 @@ struct AttnArgs {
   float* part;        // [B*H][splits][2 + d] partials of split (b, g) pairs
   int splits;         // partial slots per (b, h)
   int kvh;            // 0: idx [B][max_k], count [B] shared by the KV heads; 1: idx [B][Hkv][max_k], count [B][Hkv]
+  int Gs, hoff;       // as in ScoreArgs: heads g * Gs + hoff + [0, G) of KV head g
   unsigned* err;
 };
 
@@ -159,6 +166,8 @@ cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
 int attn_batch_tokens();
 int attn_max_batch();
 int attn_max_segments(int max_k);
-cudaError_t launch_sparse_attn(const AttnArgs& a, int dtype, int G, int grid, cudaStream_t st);
+// The attention kernel for one pass of G heads per KV head, and (combine)
+// the merge of split partials over all heads.
+cudaError_t launch_sparse_attn(const AttnArgs& a, int dtype, int G, int grid, bool combine, cudaStream_t st);
 
 }  // namespace hill

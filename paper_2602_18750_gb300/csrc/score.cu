@@ -245,7 +245,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
 #pragma unroll
     for (int r = 0; r < kMaxNg; ++r) {
       const bool has = r < ng && grp < G;
-      const int64_t row = has ? (int64_t)b * a.q_sb + (int64_t)((warp + r * kNW) * G + grp) * a.q_sh : 0;
+      const int64_t row = has ? (int64_t)b * a.q_sb + (int64_t)((warp + r * kNW) * a.Gs + a.hoff + grp) * a.q_sh : 0;
       if constexpr (F8) {
         const auto* qh = static_cast<const uint16_t*>(a.q) + row;
         float v[4][8];
@@ -316,7 +316,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
         }
         const int hl = 2 * tig + c;
         if (grp == 0 && hl < G)
-          a.partials[((int64_t)cur_b * a.nslot + cur_slot) * H + g * G + hl] = make_float2(m, l);
+          a.partials[((int64_t)cur_b * a.nslot + cur_slot) * H + g * a.Gs + a.hoff + hl] = make_float2(m, l);
       }
     }
   };
@@ -422,7 +422,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
             if (tig == 0 && t < nv) {
               const int64_t o = ((int64_t)b * Hkv + g) * cap + j0 + t;
               const float val = v * kInvSqrtD;
-              if (a.scores) a.scores[o] = val;
+              if (a.scores) a.scores[o] = a.raw_add ? a.scores[o] + val : val;
               if (a.accum) a.accum[o] += val;
             }
           } else {
@@ -430,7 +430,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
           }
         }
       } else {
-        float* lg = a.logits + ((int64_t)b * H + g * G) * cap + j0;
+        float* lg = a.logits + ((int64_t)b * H + g * a.Gs + a.hoff) * cap + j0;
 #pragma unroll
         for (int c = 0; c < kCols; ++c) {
           const int hl = 2 * tig + c;
@@ -466,7 +466,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
         for (int w = 0; w < kNW; ++w) sum += rb[w * kT + lane];
         sum *= kInvSqrtD;
         const int64_t o = (int64_t)b * cap + j0 + lane;
-        if (a.scores) a.scores[o] = sum;
+        if (a.scores) a.scores[o] = a.raw_add ? a.scores[o] + sum : sum;
         if (a.accum) a.accum[o] += sum;
       }
     } else if (!ok) {

@@ -83,7 +83,8 @@ def test_host_validation_without_device(lib):
     assert _step(lib, _desc(dtype=7)) == INV
     assert _step(lib, _desc(k_sn=100)) == INV                            # not 16-byte rows
     assert _step(lib, _desc(head_dim=64, q_sh=64)) == UNS
-    assert _step(lib, _desc(num_q_heads=32, num_kv_heads=2)) == UNS      # G = 16
+    assert _step(lib, _desc(num_q_heads=24, num_kv_heads=2)) == UNS      # G = 12
+    assert _step(lib, _desc(num_q_heads=64, num_kv_heads=1)) == UNS      # G = 64
     assert _step(lib, _desc(), max_k=-1) == INV
     assert _step(lib, _desc(), q=None) == INV
     assert _step(lib, _desc(), lens=None) == INV

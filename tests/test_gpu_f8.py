@@ -86,6 +86,7 @@ SHAPES = [
     (2, 32, 8, 700, [700, 1]),
     (2, 8, 1, 300, [300, 299]),
     (4, 16, 2, 129, [129, 0, 64, 95]),
+    (2, 32, 1, 700, [700, 333]),   # 32 query heads on one KV head
 ]
 
 

@@ -36,6 +36,8 @@ SHAPES = [
     (2, 32, 8, 600, [600, 257], [120, 51]),
     (2, 8, 1, 300, [300, 299], [30, 299]),
     (4, 16, 2, 129, [129, 0, 64, 95], [13, 3, 64, 0]),
+    (2, 32, 2, 400, [400, 177], [40, 17]),   # 16 query heads per KV head
+    (2, 32, 1, 300, [300, 123], [30, 12]),   # MQA: one KV head, 32 query heads
 ]
 
 

@@ -54,6 +54,9 @@ SHAPES = [
     # fewer query heads than one warp of the normalisation combines
     (2, 2, 1, 300, [300, 150], [30, 15]),
     (2, 1, 1, 257, [257, 100], [20, 100]),
+    # groups of more than 8 query heads per KV head (MQA-like), run in passes of 8
+    (2, 32, 1, 700, [700, 333], [70, 33]),
+    (2, 32, 2, 500, [500, 260], [50, 26]),
 ]
 
 
