@@ -43,9 +43,12 @@
  *   generated this step (the caller appends its K/V first); it is clamped to
  *   [0, cap] on the device.  Entries of scores/accum at j >= lens[b] are not
  *   touched.  k[b] is clamped to [0, lens[b]].
- * - Supported: head_dim 128; H / Hkv in {1, 2, 4, 8, 16, 32} (groups of 16 or
- *   32 query heads are scored and attended in passes of 8 over the same KV
- *   rows); fp16 or bf16 q/K/V.
+ * - Supported: head_dim 128; any H and Hkv with H a multiple of Hkv (MHA,
+ *   GQA with any group size G = H / Hkv, MQA); B <= 512; fp16 or bf16 q/K/V.
+ *   Groups of more than 8 query heads are scored and attended in passes of at
+ *   most 8 over the same KV rows, and more than 32 KV heads are scored in
+ *   passes of at most 32 (e.g. 40 KV heads: two passes of 20), each pass
+ *   streaming only its own heads' keys.
  */
 #ifndef HILL_H_
 #define HILL_H_

@@ -147,11 +147,10 @@ hill_status check_desc(const hill_desc* d) {
       !stride_ok(d->k_sn) || !stride_ok(d->v_sb) || !stride_ok(d->v_sh) || !stride_ok(d->v_sn))
     return HILL_ERR_INVALID_ARG;
   if (d->head_dim != kHeadDim) return HILL_ERR_UNSUPPORTED;
-  const int G = d->num_q_heads / d->num_kv_heads;
-  // groups of more than 8 query heads per KV head (MQA-like) run in passes of 8
-  if (G != 1 && G != 2 && G != 4 && G != 8 && G != 16 && G != 32) return HILL_ERR_UNSUPPORTED;
+  // any group size G = H / Hkv and any number of KV heads: groups of more
+  // than 8 query heads and more than score_max_kv_heads() KV heads run in
+  // passes (head_passes)
   if (d->batch > score_max_batch() || d->batch > attn_max_batch()) return HILL_ERR_UNSUPPORTED;
-  if (d->num_kv_heads > score_max_kv_heads(G > 8 ? 8 : G)) return HILL_ERR_UNSUPPORTED;
   // the selection keeps a sequence's keys on chip across at most 8 CTAs
   if (select_smem_bytes(d->capacity, select_cluster_size(d->capacity)) > 220 * 1024)
     return HILL_ERR_UNSUPPORTED;
@@ -206,6 +205,33 @@ unsigned char* ws_base(void* ws) {
 
 hill_status from_cuda(cudaError_t e) { return e == cudaSuccess ? HILL_OK : HILL_ERR_CUDA; }
 
+// The launches a scoring or attention call makes over the heads: passes of
+// at most score_max_kv_heads() KV heads (balanced), times passes of at most
+// 8 query heads of each group (the last one takes the rest).  f(goff, nkv,
+// hoff, Gn, first) is called once per pass.
+int pow2_at_least(int n) {
+  int p = 1;
+  while (p < n) p <<= 1;
+  return p;
+}
+
+template <typename F>
+hill_status head_passes(const hill_desc* d, bool kv_split, F&& f) {
+  const int Hkv = d->num_kv_heads, G = d->num_q_heads / d->num_kv_heads;
+  const int cap_kv = score_max_kv_heads();
+  const int kp = kv_split ? (Hkv + cap_kv - 1) / cap_kv : 1;
+  bool first = true;
+  for (int p = 0; p < kp; ++p) {
+    const int g0 = (int)((int64_t)p * Hkv / kp), g1 = (int)((int64_t)(p + 1) * Hkv / kp);
+    for (int h0 = 0; h0 < G; h0 += 8) {
+      const hill_status s = f(g0, g1 - g0, h0, std::min(8, G - h0), first);
+      if (s != HILL_OK) return s;
+      first = false;
+    }
+  }
+  return HILL_OK;
+}
+
 hill_status run_score(const hill_desc* d, const void* q, const void* k, const int32_t* lens, int mode,
                       float* scores, float* accum, unsigned char* base, const Layout& L,
                       const DeviceInfo& di, cudaStream_t st, uint32_t* hist0 = nullptr, int recent = 0,
@@ -244,16 +270,19 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
     a.hist0 = hist0;
     a.hist0_words = (int64_t)d->batch * select_hist_bins();
   }
-  // a group of G > 8 query heads is scored in G / 8 passes over the same keys,
-  // 8 heads each (RAW passes after the first add their sums)
-  const int GP = G > 8 ? 8 : G;
+  // groups of more than 8 query heads are scored in passes over the same
+  // keys, and more than score_max_kv_heads() KV heads in passes over their
+  // own keys (RAW passes after the first add their sums); the kernel's group
+  // template is the power of two at or above the pass's heads
   a.Gs = G;
-  hill_status s = HILL_OK;
-  for (int p = 0; p < G / GP && s == HILL_OK; ++p) {
-    a.hoff = p * GP;
-    a.raw_add = p > 0 ? 1 : 0;
-    s = from_cuda(counted(launch_score(a, d->dtype, GP, raw, f8, L.score_grid, st), 1));
-  }
+  hill_status s = head_passes(d, true, [&](int goff, int nkv, int hoff, int Gn, bool first) {
+    a.goff = goff;
+    a.nkv = nkv;
+    a.hoff = hoff;
+    a.Gn = Gn;
+    a.raw_add = first ? 0 : 1;
+    return from_cuda(counted(launch_score(a, d->dtype, pow2_at_least(Gn), raw, f8, L.score_grid, st), 1));
+  });
   if (s != HILL_OK || raw) return s;
   FinalizeArgs f{};
   f.logits = a.logits;
@@ -328,18 +357,17 @@ hill_status run_attn(const hill_desc* d, const void* q, const void* k, const voi
   a.splits = L.splits;
   a.kvh = kvh ? 1 : 0;
   a.err = di.err;
-  // G > 8 query heads per KV head: passes of 8 heads over the same selected
-  // rows, then one merge of the split partials over all heads
+  // G > 8 query heads per KV head: passes of at most 8 heads over the same
+  // selected rows, then one merge of the split partials over all heads
   const int G = d->num_q_heads / d->num_kv_heads;
-  const int GP = G > 8 ? 8 : G;
   a.Gs = G;
-  for (int p = 0; p < G / GP; ++p) {
-    a.hoff = p * GP;
-    const bool last = p == G / GP - 1;
-    hill_status s = from_cuda(counted(launch_sparse_attn(a, d->dtype, GP, L.attn_grid, last, st), last ? 2 : 1));
-    if (s != HILL_OK) return s;
-  }
-  return HILL_OK;
+  return head_passes(d, false, [&](int, int, int hoff, int Gn, bool) {
+    a.hoff = hoff;
+    a.Gn = Gn;
+    const bool last = hoff + Gn == G;
+    return from_cuda(
+        counted(launch_sparse_attn(a, d->dtype, pow2_at_least(Gn), L.attn_grid, last, st), last ? 2 : 1));
+  });
 }
 
 }  // namespace

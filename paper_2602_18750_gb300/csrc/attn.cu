@@ -202,11 +202,13 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   advance(pl);
 
   // mma.sync fragments: grp = lane/4, tig = lane%4.  S accumulators: row grp
-  // = query head grp of the group (rows >= G and 8..15 are zero), columns =
+  // = query head grp of the group (rows >= Gn and 8..15 are zero; Gn = G
+  // unless G is 4 or 8 and the group has 3, or 5 to 7 heads), columns =
   // tokens nb*8 + 2*tig + {0,1}.  O^T accumulators: rows = dims db*16 + grp
   // (+8), columns = heads 2*tig, 2*tig + 1.
   const int grp = lane >> 2, tig = lane & 3;
-  const bool head_ok = grp < G;
+  const int Gn = G <= 2 ? G : a.Gn;
+  const bool head_ok = grp < Gn;
   const int hA = 2 * tig, hB = 2 * tig + 1;   // heads of this lane's O^T columns
   float m_run = -INFINITY, l_run = 0.f;       // softmax state of head grp (base 2)
   float oacc[8][4];
@@ -243,7 +245,7 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
 #pragma unroll
     for (int c = 0; c < 2; ++c) {
       const int hl = c ? hB : hA;
-      if (hl >= G) continue;
+      if (hl >= Gn) continue;
       const float m = c ? mB : mA, l = c ? lB : lA;
       const int h = cg * a.Gs + a.hoff + hl;
       if (whole) {

@@ -28,12 +28,14 @@ struct ScoreArgs {
   float2* partials;   // ATTN: [B][nslot][H] (max, sum 2^(z2 - max)), base-2 logits z2 = z * log2 e
   int nslot;          // = grid size of the launch
   int kvh;            // RAW with per-KV-head selection: scores/accum [B][Hkv][cap], summed over each group only
-  // Query heads per KV head in the data (Gs) and the first one this launch
-  // handles (hoff): a launch covers heads g * Gs + hoff + [0, G) of every KV
-  // head g.  Gs = G, hoff = 0 except when a group of more than 8 heads is
-  // scored in passes of 8; then RAW passes after the first add to scores
-  // (raw_add) instead of storing.
-  int Gs, hoff, raw_add;
+  // Query heads per KV head in the data (Gs), the first one this launch
+  // handles (hoff) and how many (Gn, at most the kernel's template group G,
+  // the rows past Gn being zero): a launch covers heads g * Gs + hoff +
+  // [0, Gn) of the KV heads g in [goff, goff + nkv).  Groups of more than 8
+  // heads are scored in passes of at most 8, and more than 32 KV heads in
+  // passes of at most 32; RAW passes after the first add to scores (raw_add)
+  // instead of storing.
+  int Gs, hoff, Gn, goff, nkv, raw_add;
   uint32_t* hist0;    // optional: zero-filled here (hist0_words words) for the normalisation to count into
   int64_t hist0_words;
   unsigned* err;
@@ -90,7 +92,7 @@ struct AttnArgs {
   float* part;        // [B*H][splits][2 + d] partials of split (b, g) pairs
   int splits;         // partial slots per (b, h)
   int kvh;            // 0: idx [B][max_k], count [B] shared by the KV heads; 1: idx [B][Hkv][max_k], count [B][Hkv]
-  int Gs, hoff;       // as in ScoreArgs: heads g * Gs + hoff + [0, G) of KV head g
+  int Gs, hoff, Gn;   // as in ScoreArgs: heads g * Gs + hoff + [0, Gn) of KV head g
   unsigned* err;
 };
 
@@ -145,7 +147,7 @@ size_t score_smem_bytes(int G, bool f8);
 int score_tile_tokens();
 int score_warps();
 int score_max_batch();
-int score_max_kv_heads(int G);
+int score_max_kv_heads();
 cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8, int grid, cudaStream_t st);
 // Launches the normalisation (one or two kernels: *kernels is set to the count).
 cudaError_t launch_attn_finalize(const FinalizeArgs& a, int sms, cudaStream_t st, int* kernels);

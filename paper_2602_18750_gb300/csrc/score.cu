@@ -81,7 +81,7 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 }
 
 // Position of a warp in its own stage sequence: item (global tile index), r
-// (its r-th KV head of that item, g = warp + r * kNW) and b (the item's
+// (its r-th KV head of that item, g = goff + warp + r * kNW) and b (the item's
 // sequence, advanced incrementally).
 struct Cursor {
   int item, r, b;
@@ -95,6 +95,9 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   constexpr int kStages = Cfg::kStages;
   // accumulator columns that can hold a head of the group: 2*tig (+1 when G > 1)
   constexpr int kCols = G >= 2 ? 2 : 1;
+  // heads of the group this launch handles (G itself unless G is 4 or 8 and
+  // the group is 3, or 5 to 7 heads: the query rows past Gn are zero)
+  const int Gn = G <= 2 ? G : a.Gn;
 
   extern __shared__ unsigned char smem_raw[];
   const uint32_t raw_addr = smem_addr(smem_raw);
@@ -145,7 +148,8 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   const int n_items = tstart[B];
   const int per = (n_items + gridDim.x - 1) / gridDim.x;     // items per CTA
   const int it_lo = min(n_items, (int)blockIdx.x * per), it_hi = min(n_items, it_lo + per);
-  const int ng = (Hkv - warp + kNW - 1) / kNW;   // KV heads of this warp per tile (0 .. kMaxNg)
+  // KV heads of this warp per tile (0 .. kMaxNg): goff + warp + r * kNW for r < ng
+  const int ng = (a.nkv - warp + kNW - 1) / kNW;
 
   const uint64_t pol = l2_evict_first_policy();
   const uint32_t stage0 = base_addr + warp * kSW * kSlotBytes;
@@ -163,7 +167,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   // lane 0: load the K tile of position c into slot s
   auto issue = [&](const Cursor& c, uint32_t s) {
     const int j0 = (c.item - tstart[c.b]) * kT;
-    const int g = warp + c.r * kNW;
+    const int g = a.goff + warp + c.r * kNW;
     const uint32_t fb = bar0 + s * 8;
     const uint32_t dst = stage0 + s * kSlotBytes;
     // tensor-map coordinates: dimension 0 is d, the others are ordered by stride
@@ -202,7 +206,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
       Cursor lc = pc;
       for (int u = 0; u < kL2Ahead && lc.item < it_hi; ++u) {
         const int j0 = (lc.item - tstart[lc.b]) * kT;
-        const int g = warp + lc.r * kNW;
+        const int g = a.goff + warp + lc.r * kNW;
         const int c1 = a.kdim_tok == 1 ? j0 : (a.kdim_head == 1 ? g : lc.b);
         const int c2 = a.kdim_tok == 2 ? j0 : (a.kdim_head == 2 ? g : lc.b);
         const int c3 = a.kdim_tok == 3 ? j0 : (a.kdim_head == 3 ? g : lc.b);
@@ -235,7 +239,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   int cur_b = -1, cur_slot = 0;
 
   // q of this warp's heads for the current sequence, as mma B fragments:
-  // column grp is query head g*G + grp (zero for grp >= G), k = 16*kb + 2*tig (+8)
+  // column grp is query head g*Gs + hoff + grp (zero for grp >= Gn), k = 16*kb + 2*tig (+8)
   // F8: the same rows cast to E4M3 with one scale per head, as m16n8k32 B
   // fragments (k = 32*kb + 4*tig .. +3, and +16), and the scales of this
   // lane's accumulator columns (heads 2*tig and 2*tig + 1)
@@ -244,8 +248,9 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   auto load_q = [&](int b) {
 #pragma unroll
     for (int r = 0; r < kMaxNg; ++r) {
-      const bool has = r < ng && grp < G;
-      const int64_t row = has ? (int64_t)b * a.q_sb + (int64_t)((warp + r * kNW) * a.Gs + a.hoff + grp) * a.q_sh : 0;
+      const bool has = r < ng && grp < Gn;
+      const int64_t row =
+          has ? (int64_t)b * a.q_sb + (int64_t)((a.goff + warp + r * kNW) * a.Gs + a.hoff + grp) * a.q_sh : 0;
       if constexpr (F8) {
         const auto* qh = static_cast<const uint16_t*>(a.q) + row;
         float v[4][8];
@@ -302,7 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
 #pragma unroll
     for (int r = 0; r < kMaxNg; ++r) {
       if (r >= ng) break;
-      const int g = warp + r * kNW;
+      const int g = a.goff + warp + r * kNW;
 #pragma unroll
       for (int c = 0; c < kCols; ++c) {
         float m = st_m[r][c], l = st_l[r][c];
@@ -315,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
           m = mn;
         }
         const int hl = 2 * tig + c;
-        if (grp == 0 && hl < G)
+        if (grp == 0 && hl < Gn)
           a.partials[((int64_t)cur_b * a.nslot + cur_slot) * H + g * a.Gs + a.hoff + hl] = make_float2(m, l);
       }
     }
@@ -340,7 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
 #pragma unroll
     for (int r = 0; r < kMaxNg; ++r) {
       if (r >= ng || !ok) break;
-      const int g = warp + r * kNW;
+      const int g = a.goff + warp + r * kNW;
       // every lane waits; the warp goes on only if all of them saw the phase
       // complete, so it takes the same path and its shuffles stay converged
       if (!__all_sync(0xffffffffu, mbar_wait(bar0 + cs * 8, cph, a.err))) {
@@ -407,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
       }
 
       // acc[mb][c] = token mb*16 + grp, column 2*tig + c; acc[mb][2 + c] = token
-      // mb*16 + grp + 8.  Columns >= G are zero (their q fragments are zero).
+      // mb*16 + grp + 8.  Columns >= Gn are zero (their q fragments are zero).
       if constexpr (RAW) {
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
@@ -440,7 +445,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
             const int mb = u >> 1, e = (u & 1) * 2 + c;
             const int t = mb * 16 + grp + (u & 1) * 8;
             z[u] = t < nv ? acc[mb][e] * kLog2eInvSqrtD : -INFINITY;
-            if (t < nv && hl < G) lg[(int64_t)hl * cap + t] = z[u];
+            if (t < nv && hl < Gn) lg[(int64_t)hl * cap + t] = z[u];
           }
           const float mn = fmaxf(st_m[r][c], fmaxf(fmaxf(z[0], z[1]), fmaxf(z[2], z[3])));
           st_l[r][c] = st_l[r][c] * ex2(st_m[r][c] - mn) +
@@ -542,9 +547,11 @@ __device__ __forceinline__ void combine_partials(const FinalizeArgs& a, int b, i
 }
 
 // STATS: the per-head (max, 1/sum) come from hill_attn_stats_kernel instead of
-// every CTA combining the partials itself (long sequences: many CTAs).
-template <bool STATS>
-__global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(FinalizeArgs a) {
+// every CTA combining the partials itself (long sequences: many CTAs).  KVH:
+// per-KV-head importance (a.kvh), a variant of its own so that its group sums
+// do not weigh on the registers of the plain kernel.
+template <bool STATS, bool KVH>
+__global__ void __launch_bounds__(kFinThreads, STATS ? 4 : 2) hill_attn_finalize_kernel(FinalizeArgs a) {
   extern __shared__ float fsm[];
   float* mh = fsm;            // [H]
   float* il = fsm + a.H;      // [H]
@@ -606,11 +613,12 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
   if (a.hist0)
     for (int i = threadIdx.x; i < kHistBins; i += kFinThreads) hcount[i] = 0u;
   __syncthreads();
-  if (valid && a.kvh) {
+  if (KVH && valid) {
     // per-KV-head importance: the sum over each group of G query heads,
     // stored as soon as the group is complete (heads of a group are adjacent)
-    const int gm = a.H / a.Hkv - 1;   // G - 1 (G is a power of two)
-    auto put = [&](int g, float v) {
+    const int G = a.H / a.Hkv;
+    int g = 0, in_g = 0;   // the group being summed and its heads so far
+    auto put = [&](float v) {
       const int64_t o = ((int64_t)b * a.Hkv + g) * a.cap + j;
       if (a.scores) a.scores[o] = v;
       if (a.accum) a.accum[o] += v;
@@ -620,8 +628,10 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
     for (int u = 0; u < kFinZReg; ++u)
       if (u < a.H) {
         sg += ex2(zr[u] - mh[u]) * il[u];
-        if (((u + 1) & gm) == 0) {
-          put(u / (gm + 1), sg);
+        if (++in_g == G) {
+          put(sg);
+          ++g;
+          in_g = 0;
           sg = 0.f;
         }
       }
@@ -633,13 +643,15 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
       for (int u = 0; u < 16; ++u)
         if (h + u < a.H) {
           sg += ex2(z[u] - mh[h + u]) * il[h + u];
-          if (((h + u + 1) & gm) == 0) {
-            put((h + u) / (gm + 1), sg);
+          if (++in_g == G) {
+            put(sg);
+            ++g;
+            in_g = 0;
             sg = 0.f;
           }
         }
     }
-  } else if (valid) {
+  } else if (!KVH && valid) {
     float s = 0.f;
 #pragma unroll
     for (int u = 0; u < kFinZReg; ++u)
@@ -675,7 +687,7 @@ __global__ void __launch_bounds__(kFinThreads) hill_attn_finalize_kernel(Finaliz
 // Combine the per-CTA (max, sum) partials of one (b, h) into its softmax
 // statistics (max, 1 / sum) in the base-2 scale: one warp per pair, each lane
 // taking every 32nd partial with a running maximum, the lanes then merged by
-// shuffles.  Used ahead of hill_attn_finalize_kernel<true> when the
+// shuffles.  Used ahead of hill_attn_finalize_kernel<true, *> when the
 // normalisation has many CTAs per sequence.
 constexpr int kStatsWarps = 8;
 constexpr int kStatsPer = 8;   // partials per lane whose loads are in flight together
@@ -774,10 +786,7 @@ size_t score_smem_bytes(int G, bool f8) {
 int score_tile_tokens() { return kT; }
 int score_warps() { return kNW; }
 int score_max_batch() { return kMaxBatchSmem; }
-int score_max_kv_heads(int G) {
-  (void)G;
-  return kMaxNg * kNW;
-}
+int score_max_kv_heads() { return kMaxNg * kNW; }
 
 cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8, int grid, cudaStream_t st) {
   if (dtype == 0) return f8 ? launch_score_m<0, true>(a, G, raw, grid, st) : launch_score_m<0, false>(a, G, raw, grid, st);
@@ -795,10 +804,12 @@ cudaError_t launch_attn_finalize(const FinalizeArgs& a, int sms, cudaStream_t st
     cudaError_t e = launch_pdl(hill_attn_stats_kernel, dim3((pairs + kStatsWarps - 1) / kStatsWarps),
                                dim3(kStatsWarps * 32), 0, st, 0, a);
     if (e != cudaSuccess) return e;
-    return launch_pdl(hill_attn_finalize_kernel<true>, grid, dim3(kFinThreads), smem, st, 0, a);
+    return a.kvh ? launch_pdl(hill_attn_finalize_kernel<true, true>, grid, dim3(kFinThreads), smem, st, 0, a)
+                 : launch_pdl(hill_attn_finalize_kernel<true, false>, grid, dim3(kFinThreads), smem, st, 0, a);
   }
   *kernels = 1;
-  return launch_pdl(hill_attn_finalize_kernel<false>, grid, dim3(kFinThreads), smem, st, 0, a);
+  return a.kvh ? launch_pdl(hill_attn_finalize_kernel<false, true>, grid, dim3(kFinThreads), smem, st, 0, a)
+               : launch_pdl(hill_attn_finalize_kernel<false, false>, grid, dim3(kFinThreads), smem, st, 0, a);
 }
 
 }  // namespace hill

@@ -83,8 +83,14 @@ def test_host_validation_without_device(lib):
     assert _step(lib, _desc(dtype=7)) == INV
     assert _step(lib, _desc(k_sn=100)) == INV                            # not 16-byte rows
     assert _step(lib, _desc(head_dim=64, q_sh=64)) == UNS
-    assert _step(lib, _desc(num_q_heads=24, num_kv_heads=2)) == UNS      # G = 12
-    assert _step(lib, _desc(num_q_heads=64, num_kv_heads=1)) == UNS      # G = 64
+    assert _step(lib, _desc(batch=513)) == UNS                            # above the per-CTA tables
+    # any group size and any number of KV heads pass the host checks (the call
+    # then fails only for want of a device here)
+    from paper_2602_18750_gb300.hill import HILL_ERR_CUDA as CUDA
+    for hq, hkv in [(24, 2), (64, 1), (28, 4), (12, 4), (40, 40), (80, 10)]:
+        d = _desc(num_q_heads=hq, num_kv_heads=hkv, q_sb=hq * 128,
+                  k_sb=hkv * 64 * 128, v_sb=hkv * 64 * 128)
+        assert _step(lib, d) == CUDA, (hq, hkv)
     assert _step(lib, _desc(), max_k=-1) == INV
     assert _step(lib, _desc(), q=None) == INV
     assert _step(lib, _desc(), lens=None) == INV

@@ -87,6 +87,8 @@ SHAPES = [
     (2, 8, 1, 300, [300, 299]),
     (4, 16, 2, 129, [129, 0, 64, 95]),
     (2, 32, 1, 700, [700, 333]),   # 32 query heads on one KV head
+    (2, 28, 4, 300, [300, 150]),   # 7 query heads per KV head
+    (2, 40, 40, 200, [200, 77]),   # 40 KV heads: two scoring passes
 ]
 
 
@@ -96,6 +98,26 @@ SHAPES = [
 def test_score_f8_matches_oracle(H, oracle_mod, mode, dtype, shape):
     B, Hq, Hkv, cap, lens = shape
     q, K, V, lens_t = inputs.random_case(B, Hq, Hkv, 128, cap, lens, dtype=dtype, seed=cap + Hq)
+    q, K, lens_t = q.cuda(), K.cuda(), lens_t.cuda()
+    desc = H.make_desc(q, K)
+    k8, ks = _shadow(H, desc, K, lens)
+    ws = H.alloc_workspace(desc, mode, 0)
+    s = torch.zeros(B, cap, device="cuda")
+    H.hill_score_f8(desc, q, k8, ks, lens_t, mode, s, ws=ws)
+    H.hill_sync_status()
+    codes, scale = oracle_mod.quantize_rows(K.cpu())
+    z8 = oracle_mod.logits_q8(q.cpu(), codes, scale, lens)
+    check_scores(s.cpu().numpy(), oracle_mod.scores(mode, z8, lens), lens)
+
+
+@pytest.mark.parametrize("mode", [ATTN, RAW])
+def test_score_f8_long(H, oracle_mod, mode):
+    """Long sequences: many tiles per scoring CTA, and (ATTN) the
+    normalisation with more than two CTAs per SM, which first combines the
+    partials once per (sequence, head)."""
+    B, Hq, Hkv, cap = 2, 8, 8, 40000
+    lens = [40000, 23457]
+    q, K, V, lens_t = inputs.random_case(B, Hq, Hkv, 128, cap, lens, dtype=torch.float16, seed=404)
     q, K, lens_t = q.cuda(), K.cuda(), lens_t.cuda()
     desc = H.make_desc(q, K)
     k8, ks = _shadow(H, desc, K, lens)

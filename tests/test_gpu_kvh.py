@@ -38,6 +38,9 @@ SHAPES = [
     (4, 16, 2, 129, [129, 0, 64, 95], [13, 3, 64, 0]),
     (2, 32, 2, 400, [400, 177], [40, 17]),   # 16 query heads per KV head
     (2, 32, 1, 300, [300, 123], [30, 12]),   # MQA: one KV head, 32 query heads
+    (2, 28, 4, 300, [300, 77], [30, 7]),     # 7 query heads per KV head
+    (2, 12, 1, 200, [200, 64], [20, 6]),     # 12 = 8 + 4 heads on one KV head
+    (1, 40, 40, 200, [200], [40]),           # 40 KV heads: two scoring passes
 ]
 
 

@@ -57,6 +57,14 @@ SHAPES = [
     # groups of more than 8 query heads per KV head (MQA-like), run in passes of 8
     (2, 32, 1, 700, [700, 333], [70, 33]),
     (2, 32, 2, 500, [500, 260], [50, 26]),
+    # group sizes that are not powers of two (the kernels' power-of-two group
+    # templates with the extra query rows zero), and one of 12 = 8 + 4 heads
+    (2, 12, 4, 300, [300, 171], [30, 17]),
+    (2, 28, 4, 400, [400, 95], [40, 9]),
+    (1, 24, 2, 257, [257], [25]),
+    # more KV heads than one scoring launch holds (40, as LLaMA-13B): two
+    # passes of 20 KV heads
+    (2, 40, 40, 300, [300, 130], [60, 26]),
 ]
 
 
