@@ -244,7 +244,8 @@ const char* hill_status_string(hill_status status);
  *    before any stream capture.
  *  - A call needing more scratch than the array holds returns
  *    HILL_ERR_WORKSPACE without launching anything.  ATTN mode needs about
- *    4*B*cap*(H + 1) + 8*B*H*(SMs + 1) bytes; RAW about 4*B*cap.
+ *    4*B*cap*(H + 1) + 8*B*H*(SMs*W + 1) bytes, W = 8 / Hkv rounded down
+ *    when Hkv <= 4 and H / Hkv >= 5, else 1; RAW about 4*B*cap.
  *  - All calls share the array, and it keeps whatever the last call left;
  *    no entry of it needs to start at zero (a call reads only what it wrote).
  *    Calls that overlap on the GPU (two streams, or two host threads without

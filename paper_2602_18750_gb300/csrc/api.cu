@@ -161,6 +161,7 @@ struct Layout {
   size_t scores, logits, partials, stats, hist0, attn_part, total;
   bool has_hist0;
   int score_grid, attn_grid, splits;
+  int score_spc;   // ATTN partial slots per scoring CTA
 };
 
 int score_grid_for(const hill_desc* d, int sms) {
@@ -175,6 +176,12 @@ Layout layout_for(const hill_desc* d, int mode, int max_k, int sms) {
   Layout L{};
   const size_t B = d->batch, H = d->num_q_heads, cap = d->capacity;
   L.score_grid = score_grid_for(d, sms);
+  // few KV heads with large groups (MQA-like): the scoring kernel deals the
+  // tiles to several warps per head, each with its own partial slot (more
+  // than score_max_kv_heads() KV heads run in passes of at least half that)
+  L.score_spc = d->num_kv_heads > score_max_kv_heads()
+                    ? 1
+                    : score_deal_warps(d->num_kv_heads, d->num_q_heads / d->num_kv_heads);
   L.attn_grid = sms;
   L.splits = attn_max_segments(max_k < 0 ? 0 : max_k);
   size_t off = 0;
@@ -183,7 +190,7 @@ Layout layout_for(const hill_desc* d, int mode, int max_k, int sms) {
   L.logits = off;
   if (mode == HILL_SCORE_ATTN) off += align_up(B * H * cap * sizeof(float));
   L.partials = off;
-  if (mode == HILL_SCORE_ATTN) off += align_up(B * (size_t)L.score_grid * H * sizeof(float2));
+  if (mode == HILL_SCORE_ATTN) off += align_up(B * (size_t)L.score_grid * L.score_spc * H * sizeof(float2));
   // combined (max, 1/sum) per (b, h), when the normalisation runs in two kernels
   L.stats = off;
   if (mode == HILL_SCORE_ATTN) off += align_up(B * H * sizeof(float2));
@@ -251,7 +258,7 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   a.k_sb = d->k_sb;
   a.k_sh = d->k_sh;
   a.k_sn = d->k_sn;
-  a.nslot = L.score_grid;
+  a.nslot = L.score_grid * L.score_spc;
   a.err = di.err;
   // kscale != NULL: k is the E4M3 shadow of the keys (asymmetric-precision scoring)
   const bool f8 = kscale != nullptr;
@@ -281,7 +288,11 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
     a.hoff = hoff;
     a.Gn = Gn;
     a.raw_add = first ? 0 : 1;
-    return from_cuda(counted(launch_score(a, d->dtype, pow2_at_least(Gn), raw, f8, L.score_grid, st), 1));
+    // the dealing kernel exists for the group template 8 (it is chosen for
+    // groups of 5 or more heads, whose passes all fit it)
+    const bool deal = L.score_spc > 1;
+    return from_cuda(
+        counted(launch_score(a, d->dtype, deal ? 8 : pow2_at_least(Gn), raw, f8, deal, L.score_grid, st), 1));
   });
   if (s != HILL_OK || raw) return s;
   FinalizeArgs f{};
@@ -291,7 +302,8 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   f.B = d->batch;
   f.H = d->num_q_heads;
   f.cap = d->capacity;
-  f.nslot = L.score_grid;
+  f.nslot = L.score_grid * L.score_spc;
+  f.spc = L.score_spc;
   f.scores = scores;
   f.accum = accum;
   f.hist0 = hist0;

@@ -26,7 +26,7 @@ struct ScoreArgs {
   float* accum;       // RAW: running importance (+=), may be NULL
   float* logits;      // ATTN: [B][H][cap]
   float2* partials;   // ATTN: [B][nslot][H] (max, sum 2^(z2 - max)), base-2 logits z2 = z * log2 e
-  int nslot;          // = grid size of the launch
+  int nslot;          // = grid size of the launch x score_deal_warps(nkv, G) (one slot per warp share)
   int kvh;            // RAW with per-KV-head selection: scores/accum [B][Hkv][cap], summed over each group only
   // Query heads per KV head in the data (Gs), the first one this launch
   // handles (hoff) and how many (Gn, at most the kernel's template group G,
@@ -46,6 +46,7 @@ struct FinalizeArgs {
   const float2* partials;
   const int32_t* lens;
   int B, H, cap, nslot;
+  int spc;            // partial slots per scoring CTA (nslot = CTAs x spc)
   float* scores;      // may be NULL when accum is given
   float* accum;       // may be NULL
   uint32_t* hist0;    // optional [B][2048]: counts of the leading 11-bit digit of the selection key
@@ -148,7 +149,13 @@ int score_tile_tokens();
 int score_warps();
 int score_max_batch();
 int score_max_kv_heads();
-cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8, int grid, cudaStream_t st);
+// Warps of the scoring kernel that share one KV head (the partial slots per
+// CTA) when a call's launches cover nkv KV heads with groups of G query heads:
+// kNW / nkv for nkv <= kNW / 2 and G >= 5, whose launches then all take the
+// dealing kernel (deal = true, group template 8); else 1.
+int score_deal_warps(int nkv, int G);
+cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8, bool deal, int grid,
+                         cudaStream_t st);
 // Launches the normalisation (one or two kernels: *kernels is set to the count).
 cudaError_t launch_attn_finalize(const FinalizeArgs& a, int sms, cudaStream_t st, int* kernels);
 

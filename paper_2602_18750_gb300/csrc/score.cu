@@ -62,7 +62,7 @@ struct ScoreCfg {
   static constexpr int kOffTab = kOffBar + kStages * 8;
   static constexpr int kOffRed = kOffTab + 2 * kTableInts * 4;
   static constexpr int kOffFlag = kOffRed + 2 * kNW * kT * 4;
-  static constexpr int kBytes = kOffFlag + 16 + 1024;        // + alignment slack
+  static constexpr int kBytes = kOffFlag + kNW * 4 + 1024;   // + alignment slack
 };
 
 constexpr int kL2Ahead = 4;   // stages per warp brought into L2 before the dependency wait
@@ -87,7 +87,7 @@ struct Cursor {
   int item, r, b;
 };
 
-template <int DT, int G, bool RAW, bool F8>
+template <int DT, int G, bool RAW, bool F8, bool DEAL>
 __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_constant__ ScoreArgs a) {
   using Cfg = ScoreCfg<G, F8>;
   constexpr int kSlotBytes = Cfg::kSlotBytes;
@@ -106,7 +106,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   int* tstart = reinterpret_cast<int*>(base + Cfg::kOffTab);          // [B+1] tile prefix
   int* slen = tstart + kTableInts;                                     // [B] clamped lengths
   float* red = reinterpret_cast<float*>(base + Cfg::kOffRed);          // [2][kNW][kT]
-  volatile int* abort_flag = reinterpret_cast<int*>(base + Cfg::kOffFlag);
+  volatile int* abort_flag = reinterpret_cast<int*>(base + Cfg::kOffFlag);   // [kNW]: one per warp group
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -115,7 +115,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) mbar_init(base_addr + Cfg::kOffBar + s * 8, 1);
     fence_barrier_init();
-    *abort_flag = 0;
+    for (int w = 0; w < kNW; ++w) abort_flag[w] = 0;
     prefetch_tmap(&a.kmap);
   }
   // Before the dependency wait this kernel reads only the inputs of the call
@@ -148,26 +148,35 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   const int n_items = tstart[B];
   const int per = (n_items + gridDim.x - 1) / gridDim.x;     // items per CTA
   const int it_lo = min(n_items, (int)blockIdx.x * per), it_hi = min(n_items, it_lo + per);
-  // KV heads of this warp per tile (0 .. kMaxNg): goff + warp + r * kNW for r < ng
-  const int ng = (a.nkv - warp + kNW - 1) / kNW;
+  // The warps' shares.  Without DEAL (W = 1) the KV heads are dealt to the
+  // warps -- warp w takes g0 + r * kNW, r < ng (0 .. kMaxNg) -- and every warp
+  // visits every item of the CTA.  With DEAL (launches of at most kNW / 2 KV
+  // heads), W = kNW / nkv warps share each head and deal the items instead:
+  // warp sub * nkv + i takes head goff + i of items it_lo + sub, + W, ...,
+  // so that every warp streams (W * nkv < kNW leaves the rest idle).
+  const int W = DEAL ? kNW / a.nkv : 1;
+  const int sub = DEAL ? warp / a.nkv : 0;
+  const int g0 = a.goff + (DEAL ? warp % a.nkv : warp);
+  const int ng = DEAL ? (warp < W * a.nkv ? 1 : 0) : (a.nkv - warp + kNW - 1) / kNW;
+  const int it0 = (DEAL && ng == 0) ? it_hi : it_lo + sub;   // this warp's first item
 
   const uint64_t pol = l2_evict_first_policy();
   const uint32_t stage0 = base_addr + warp * kSW * kSlotBytes;
   const uint32_t bar0 = base_addr + Cfg::kOffBar + warp * kSW * 8;
   const uint32_t scale0 = base_addr + Cfg::kOffScale + warp * kSW * kT * 4;   // F8 only
-  const int b_first = it_lo < it_hi ? find_seq(tstart, B, it_lo) : 0;
+  const int b_first = it0 < it_hi ? find_seq(tstart, B, it0) : 0;
 
   auto advance = [&](Cursor& c) {
     if (++c.r >= ng) {
       c.r = 0;
-      ++c.item;
+      c.item += W;
       while (c.b < B - 1 && tstart[c.b + 1] <= c.item) ++c.b;
     }
   };
   // lane 0: load the K tile of position c into slot s
   auto issue = [&](const Cursor& c, uint32_t s) {
     const int j0 = (c.item - tstart[c.b]) * kT;
-    const int g = a.goff + warp + c.r * kNW;
+    const int g = g0 + c.r * kNW;
     const uint32_t fb = bar0 + s * 8;
     const uint32_t dst = stage0 + s * kSlotBytes;
     // tensor-map coordinates: dimension 0 is d, the others are ordered by stride
@@ -187,7 +196,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   };
 
   // prologue: the first kSW stages of this warp
-  Cursor pc{it_lo, 0, b_first};
+  Cursor pc{it0, 0, b_first};
   uint32_t issued = 0, is_slot = 0;
   auto prologue = [&]() {
     if (ng > 0) {
@@ -206,7 +215,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
       Cursor lc = pc;
       for (int u = 0; u < kL2Ahead && lc.item < it_hi; ++u) {
         const int j0 = (lc.item - tstart[lc.b]) * kT;
-        const int g = a.goff + warp + lc.r * kNW;
+        const int g = g0 + lc.r * kNW;
         const int c1 = a.kdim_tok == 1 ? j0 : (a.kdim_head == 1 ? g : lc.b);
         const int c2 = a.kdim_tok == 2 ? j0 : (a.kdim_head == 2 ? g : lc.b);
         const int c3 = a.kdim_tok == 3 ? j0 : (a.kdim_head == 3 ? g : lc.b);
@@ -250,7 +259,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
     for (int r = 0; r < kMaxNg; ++r) {
       const bool has = r < ng && grp < Gn;
       const int64_t row =
-          has ? (int64_t)b * a.q_sb + (int64_t)((a.goff + warp + r * kNW) * a.Gs + a.hoff + grp) * a.q_sh : 0;
+          has ? (int64_t)b * a.q_sb + (int64_t)((g0 + r * kNW) * a.Gs + a.hoff + grp) * a.q_sh : 0;
       if constexpr (F8) {
         const auto* qh = static_cast<const uint16_t*>(a.q) + row;
         float v[4][8];
@@ -307,7 +316,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
 #pragma unroll
     for (int r = 0; r < kMaxNg; ++r) {
       if (r >= ng) break;
-      const int g = a.goff + warp + r * kNW;
+      const int g = g0 + r * kNW;
 #pragma unroll
       for (int c = 0; c < kCols; ++c) {
         float m = st_m[r][c], l = st_l[r][c];
@@ -325,8 +334,30 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
       }
     }
   };
+  // ATTN with DEAL: a warp owns one partial slot in every sequence its CTA
+  // meets, and writes a neutral one (-inf, 0) where it visited no tile of it
+  // (the normalisation skips entries whose sum is 0).  b_next: the first
+  // sequence of the CTA this warp has not written yet.
+  const int b_cta_last = it_lo < it_hi ? find_seq(tstart, B, it_hi - 1) : -1;
+  int b_next = it_lo < it_hi ? find_seq(tstart, B, it_lo) : 0;
+  auto neutral_until = [&](int b_end) {   // sequences [b_next, b_end)
+    if constexpr (!RAW && DEAL) {
+      if (ng == 0) return;
+      for (; b_next < b_end; ++b_next) {
+        if (tstart[b_next + 1] == tstart[b_next]) continue;   // empty: no slots
+        const int slot = ((int)blockIdx.x - tstart[b_next] / per) * W + sub;
+#pragma unroll
+        for (int c = 0; c < kCols; ++c) {
+          const int hl = 2 * tig + c;
+          if (grp == 0 && hl < Gn)
+            a.partials[((int64_t)b_next * a.nslot + slot) * H + g0 * a.Gs + a.hoff + hl] =
+                make_float2(-INFINITY, 0.f);
+        }
+      }
+    }
+  };
 
-  for (int item = it_lo, b = b_first; item < it_hi; ++item, ++item_no) {
+  for (int item = it0, b = b_first; item < it_hi; item += W, ++item_no) {
     while (b < B - 1 && tstart[b + 1] <= item) ++b;
     const int tile = item - tstart[b];
     const int j0 = tile * kT;
@@ -335,22 +366,25 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
 
     if (b != cur_b) {
       if (!RAW && cur_b >= 0) flush();
+      neutral_until(b);
+      b_next = b + 1;
       load_q(b);
       if (!RAW) reset_stat();
       cur_b = b;
-      // this CTA's partial slot in b: its rank among the CTAs whose ranges meet b
-      cur_slot = (int)blockIdx.x - tstart[b] / per;
+      // this warp's partial slot in b: the CTA's rank among the CTAs whose
+      // ranges meet b, times W, plus the warp's item share
+      cur_slot = ((int)blockIdx.x - tstart[b] / per) * W + sub;
     }
 
 #pragma unroll
     for (int r = 0; r < kMaxNg; ++r) {
       if (r >= ng || !ok) break;
-      const int g = a.goff + warp + r * kNW;
+      const int g = g0 + r * kNW;
       // every lane waits; the warp goes on only if all of them saw the phase
       // complete, so it takes the same path and its shuffles stay converged
       if (!__all_sync(0xffffffffu, mbar_wait(bar0 + cs * 8, cph, a.err))) {
         ok = false;
-        *abort_flag = 1;
+        abort_flag[sub] = 1;
         break;
       }
       const uint32_t sb = stage0 + cs * kSlotBytes;
@@ -455,20 +489,21 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
       }
     }
     if (RAW && !a.kvh) {
-      // sum over the warps in a fixed order, double-buffered by item; a warp
-      // whose wait timed out still reaches the barrier, and all warps then
-      // leave together
+      // sum over the warps holding the item's heads -- all kNW (W = 1), or
+      // the nkv warps of group sub -- in a fixed order, double-buffered by
+      // item; a warp whose wait timed out still reaches its group's barrier
+      // after raising the group's flag, and the group then leaves together
+      const int wg0 = DEAL ? sub * a.nkv : 0, gw = DEAL ? a.nkv : kNW;
       float* rb = red + (item_no & 1) * kNW * kT;
       if (tig == 0) {
 #pragma unroll
         for (int u = 0; u < 4; ++u) rb[warp * kT + (u >> 1) * 16 + grp + (u & 1) * 8] = rs[u];
       }
-      named_sync(1, kThreads);
-      if (*abort_flag) break;
-      if (warp == (item_no % kNW) && lane < nv) {
+      named_sync(1 + sub, gw * 32);
+      if (abort_flag[sub]) break;
+      if (warp == wg0 + item_no % gw && lane < nv) {
         float sum = 0.f;
-#pragma unroll
-        for (int w = 0; w < kNW; ++w) sum += rb[w * kT + lane];
+        for (int w = 0; w < gw; ++w) sum += rb[(wg0 + w) * kT + lane];
         sum *= kInvSqrtD;
         const int64_t o = (int64_t)b * cap + j0 + lane;
         if (a.scores) a.scores[o] = a.raw_add ? a.scores[o] + sum : sum;
@@ -479,6 +514,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
     }
   }
   if (!RAW && cur_b >= 0 && ok) flush();
+  if (ok) neutral_until(b_cta_last + 1);
   // after a timeout: give every copy this warp issued and did not consume one
   // more bounded wait before the CTA's shared memory is released
   if (!ok && lane == 0) {
@@ -585,9 +621,10 @@ __global__ void __launch_bounds__(kFinThreads, STATS ? 4 : 2) hill_attn_finalize
   }
   __syncthreads();
   const int first_item = s_first;
-  const int per = (s_total + a.nslot - 1) / a.nslot;
+  const int grid = a.nslot / a.spc;   // CTAs of the scoring launch
+  const int per = (s_total + grid - 1) / grid;
   const int items = (len + kT - 1) / kT;
-  const int ns = (first_item + items - 1) / per - first_item / per + 1;
+  const int ns = ((first_item + items - 1) / per - first_item / per + 1) * a.spc;
   pdl_wait();
   pdl_launch_dependents();
   // this token's logits of the first kFinZReg heads, loaded before the
@@ -714,8 +751,9 @@ __global__ void __launch_bounds__(kStatsWarps * 32) hill_attn_stats_kernel(Final
   int len = a.lens[b];
   len = len < 0 ? 0 : (len > a.cap ? a.cap : len);
   const int items = (len + kT - 1) / kT;
-  const int per = (t + a.nslot - 1) / a.nslot;
-  const int ns = items == 0 ? 0 : (f + items - 1) / per - f / per + 1;
+  const int grid = a.nslot / a.spc;   // CTAs of the scoring launch
+  const int per = (t + grid - 1) / grid;
+  const int ns = items == 0 ? 0 : ((f + items - 1) / per - f / per + 1) * a.spc;
   pdl_wait();
   pdl_launch_dependents();
   const float2* pb = a.partials + (int64_t)b * a.nslot * a.H + h;
@@ -746,10 +784,10 @@ __global__ void __launch_bounds__(kStatsWarps * 32) hill_attn_stats_kernel(Final
   if (lane == 0) a.stats[pair] = make_float2(m, 1.f / l);
 }
 
-template <int DT, int G, bool RAW, bool F8>
+template <int DT, int G, bool RAW, bool F8, bool DEAL>
 cudaError_t launch_score_t(const ScoreArgs& a, int grid, cudaStream_t st) {
   const size_t smem = (size_t)ScoreCfg<G, F8>::kBytes;
-  auto kern = hill_score_kernel<DT, G, RAW, F8>;
+  auto kern = hill_score_kernel<DT, G, RAW, F8, DEAL>;
   static int cache[64] = {0};
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), (int)smem, cache);
   if (e != cudaSuccess) return e;
@@ -757,19 +795,21 @@ cudaError_t launch_score_t(const ScoreArgs& a, int grid, cudaStream_t st) {
 }
 
 template <int DT, bool RAW, bool F8>
-cudaError_t launch_score_g(const ScoreArgs& a, int G, int grid, cudaStream_t st) {
+cudaError_t launch_score_g(const ScoreArgs& a, int G, bool deal, int grid, cudaStream_t st) {
+  if (deal) return G == 8 ? launch_score_t<DT, 8, RAW, F8, true>(a, grid, st) : cudaErrorInvalidValue;
   switch (G) {
-    case 1: return launch_score_t<DT, 1, RAW, F8>(a, grid, st);
-    case 2: return launch_score_t<DT, 2, RAW, F8>(a, grid, st);
-    case 4: return launch_score_t<DT, 4, RAW, F8>(a, grid, st);
-    case 8: return launch_score_t<DT, 8, RAW, F8>(a, grid, st);
+    case 1: return launch_score_t<DT, 1, RAW, F8, false>(a, grid, st);
+    case 2: return launch_score_t<DT, 2, RAW, F8, false>(a, grid, st);
+    case 4: return launch_score_t<DT, 4, RAW, F8, false>(a, grid, st);
+    case 8: return launch_score_t<DT, 8, RAW, F8, false>(a, grid, st);
   }
   return cudaErrorInvalidValue;
 }
 
 template <int DT, bool F8>
-cudaError_t launch_score_m(const ScoreArgs& a, int G, bool raw, int grid, cudaStream_t st) {
-  return raw ? launch_score_g<DT, true, F8>(a, G, grid, st) : launch_score_g<DT, false, F8>(a, G, grid, st);
+cudaError_t launch_score_m(const ScoreArgs& a, int G, bool raw, bool deal, int grid, cudaStream_t st) {
+  return raw ? launch_score_g<DT, true, F8>(a, G, deal, grid, st)
+             : launch_score_g<DT, false, F8>(a, G, deal, grid, st);
 }
 
 }  // namespace
@@ -787,10 +827,13 @@ int score_tile_tokens() { return kT; }
 int score_warps() { return kNW; }
 int score_max_batch() { return kMaxBatchSmem; }
 int score_max_kv_heads() { return kMaxNg * kNW; }
+int score_deal_warps(int nkv, int G) { return nkv <= kNW / 2 && G >= 5 ? kNW / nkv : 1; }
 
-cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8, int grid, cudaStream_t st) {
-  if (dtype == 0) return f8 ? launch_score_m<0, true>(a, G, raw, grid, st) : launch_score_m<0, false>(a, G, raw, grid, st);
-  return f8 ? launch_score_m<1, true>(a, G, raw, grid, st) : launch_score_m<1, false>(a, G, raw, grid, st);
+cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8, bool deal, int grid,
+                         cudaStream_t st) {
+  if (dtype == 0)
+    return f8 ? launch_score_m<0, true>(a, G, raw, deal, grid, st) : launch_score_m<0, false>(a, G, raw, deal, grid, st);
+  return f8 ? launch_score_m<1, true>(a, G, raw, deal, grid, st) : launch_score_m<1, false>(a, G, raw, deal, grid, st);
 }
 
 cudaError_t launch_attn_finalize(const FinalizeArgs& a, int sms, cudaStream_t st, int* kernels) {

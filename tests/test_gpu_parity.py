@@ -65,6 +65,13 @@ SHAPES = [
     # more KV heads than one scoring launch holds (40, as LLaMA-13B): two
     # passes of 20 KV heads
     (2, 40, 40, 300, [300, 130], [60, 26]),
+    # few KV heads with large groups deal the tiles to several warps per
+    # head: 3 KV heads of 5 query heads take 2 warps each (2 warps idle)
+    (3, 15, 3, 300, [300, 5, 240], [30, 5, 24]),
+    # one KV head over many short sequences: most warps of a CTA visit no
+    # tile of a sequence and leave neutral partials
+    (16, 8, 1, 100, [100, 0, 1, 31, 32, 33, 64, 65, 96, 97, 99, 2, 63, 40, 7, 100],
+     [10, 0, 1, 3, 3, 3, 6, 6, 9, 9, 9, 1, 6, 4, 1, 10]),
 ]
 
 
@@ -88,12 +95,14 @@ def test_evict_step_matches_oracle(H, oracle_mod, mode, dtype, shape):
     check_attn(ev.out.cpu().numpy(), out_ref)
 
 
+@pytest.mark.parametrize("Hkv", [8, 1])
 @pytest.mark.parametrize("dtype", [torch.float16, torch.bfloat16])
-def test_long_sequences_statistics_kernel(H, oracle_mod, dtype):
+def test_long_sequences_statistics_kernel(H, oracle_mod, dtype, Hkv):
     """Sequences long enough that the normalisation takes more than two CTAs
     per SM (2 x 157 CTAs on 152 SMs), so the per-head statistics come from
-    hill_attn_stats_kernel; accumulation over two steps included."""
-    B, Hq, Hkv, cap = 2, 8, 8, 40000
+    hill_attn_stats_kernel; accumulation over two steps included.  With one
+    KV head the scoring warps deal the tiles (8 partial slots per CTA)."""
+    B, Hq, cap = 2, 8, 40000
     lens, k = [40000, 23457], [4000, 2345]
     max_k = 4000
     accum = torch.zeros(B, cap, device="cuda")
