@@ -81,7 +81,8 @@ def test_golden_hand_derived(oracle_mod, case, dtype):
 
 
 # ---------------------------------------------------------------- logits
-@pytest.mark.parametrize("H,Hkv,d", [(8, 8, 128), (8, 2, 64), (4, 1, 128), (6, 3, 32)])
+@pytest.mark.parametrize("H,Hkv,d", [(8, 8, 128), (8, 2, 64), (4, 1, 128), (6, 3, 32),
+                                     (28, 4, 128), (12, 1, 64), (40, 40, 128)])
 @pytest.mark.parametrize("dtype", [torch.float16, torch.bfloat16])
 def test_logits_match_torch_fp64_matmul(oracle_mod, H, Hkv, d, dtype):
     B, cap = 3, 70
@@ -345,6 +346,24 @@ def test_kvh_mha_selects_each_heads_own_softmax_top(oracle_mod):
     for g in range(H):
         want = sorted(torch.topk(torch.from_numpy(z[0, g]), 7).indices.tolist())
         assert idx[0, g].tolist() == want
+
+
+@pytest.mark.parametrize("H,Hkv", [(14, 2), (12, 1)])
+def test_kvh_attn_group_sums_of_torch_softmax(oracle_mod, H, Hkv):
+    """Groups that are not a power of two (7) or above 8 heads (12): the
+    per-KV-head ATTN importance is the sum of the torch softmax rows of
+    exactly the G query heads h // G = g, each group carrying mass G."""
+    B, d, cap = 2, 64, 45
+    lens = [45, 17]
+    G = H // Hkv
+    q, K, V, _ = inputs.random_case(B, H, Hkv, d, cap, lens, seed=23)
+    z = oracle_mod.logits(q, K, lens)
+    s = oracle_mod.scores_kvh(oracle_mod.ATTN, z, lens, Hkv)
+    for b, n in enumerate(lens):
+        p = torch.softmax(torch.from_numpy(z[b, :, :n]), dim=-1).numpy()
+        for g in range(Hkv):
+            assert np.allclose(s[b, g, :n], p[g * G:(g + 1) * G].sum(0), rtol=1e-12, atol=1e-15)
+            assert np.isclose(s[b, g, :n].sum(), G, rtol=1e-12)
 
 
 def test_kvh_attention_uses_each_heads_rows(oracle_mod):
