@@ -212,16 +212,18 @@ unsigned char* ws_base(void* ws) {
 
 hill_status from_cuda(cudaError_t e) { return e == cudaSuccess ? HILL_OK : HILL_ERR_CUDA; }
 
-// The launches a scoring or attention call makes over the heads: passes of
-// at most score_max_kv_heads() KV heads (balanced), times passes of at most
-// 8 query heads of each group (the last one takes the rest).  f(goff, nkv,
-// hoff, Gn, first) is called once per pass.
+// The power of two at or above n: the kernels' group template for a pass of
+// n query heads per KV head.
 int pow2_at_least(int n) {
   int p = 1;
   while (p < n) p <<= 1;
   return p;
 }
 
+// The launches a scoring or attention call makes over the heads: passes of
+// at most score_max_kv_heads() KV heads (balanced), times passes of at most
+// 8 query heads of each group (the last one takes the rest).  f(goff, nkv,
+// hoff, Gn, first) is called once per pass.
 template <typename F>
 hill_status head_passes(const hill_desc* d, bool kv_split, F&& f) {
   const int Hkv = d->num_kv_heads, G = d->num_q_heads / d->num_kv_heads;
