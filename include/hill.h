@@ -127,11 +127,13 @@ hill_status hill_gather_sparse_attn(const hill_desc* desc, const void* q, const 
                                     int32_t max_k, float* out, void* ws, size_t ws_bytes,
                                     void* stream);
 
-/* The whole step for one layer: hill_score, then hill_topk_select on accum
- * (if given) else on this step's scores, then (if out != NULL)
- * hill_gather_sparse_attn over the selection.  scores may be NULL (then the
- * step's scores live in the workspace).  Results equal those of the three
- * separate calls. */
+/* The whole step for one layer, in the order of the evaluation workflow of
+ * Sec. 4.1 (steps 4-6: score the cached keys against the current query,
+ * keep the top-alpha critical tokens, attend over those only): hill_score,
+ * then hill_topk_select on accum (if given) else on this step's scores, then
+ * (if out != NULL) hill_gather_sparse_attn over the selection.  scores may be
+ * NULL (then the step's scores live in the workspace).  Results equal those
+ * of the three separate calls. */
 hill_status hill_evict_step(const hill_desc* desc, const void* q, const void* k_cache,
                             const void* v_cache, const int32_t* lens, const int32_t* k,
                             int32_t max_k, hill_score_mode mode, float* accum, float* scores,
@@ -243,9 +245,12 @@ const char* hill_status_string(hill_status status);
  *    (cudaGetSymbolAddress, no allocation); make that first call on a device
  *    before any stream capture.
  *  - A call needing more scratch than the array holds returns
- *    HILL_ERR_WORKSPACE without launching anything.  ATTN mode needs about
- *    4*B*cap*(H + 1) + 8*B*H*(SMs*W + 1) bytes, W = 8 / Hkv rounded down
- *    when Hkv <= 4 and H / Hkv >= 5, else 1; RAW about 4*B*cap.
+ *    HILL_ERR_WORKSPACE without launching anything.  ATTN mode needs
+ *    4*B*H*cap bytes of logits, 8*B*H*P bytes of softmax partials and
+ *    8*B*H bytes of statistics, each rounded up to 256 bytes; P = min(SMs,
+ *    B * ceil(cap / 32)) * W partial slots, W = 8 / Hkv rounded down when
+ *    Hkv <= 4 and H / Hkv >= 5, else 1 (SMs = the device's multiprocessor
+ *    count).  RAW mode needs none.
  *  - All calls share the array, and it keeps whatever the last call left;
  *    no entry of it needs to start at zero (a call reads only what it wrote).
  *    Calls that overlap on the GPU (two streams, or two host threads without

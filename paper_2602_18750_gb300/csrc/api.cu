@@ -172,7 +172,10 @@ int score_grid_for(const hill_desc* d, int sms) {
   return g < 1 ? 1 : (int)g;
 }
 
-Layout layout_for(const hill_desc* d, int mode, int max_k, int sms) {
+// Workspace regions of a call.  score_only: hill_score and its variants,
+// which write the caller's scores and run no selection or attention, need
+// only the ATTN normalisation's logits, partials and statistics.
+Layout layout_for(const hill_desc* d, int mode, int max_k, int sms, bool score_only = false) {
   Layout L{};
   const size_t B = d->batch, H = d->num_q_heads, cap = d->capacity;
   L.score_grid = score_grid_for(d, sms);
@@ -183,10 +186,11 @@ Layout layout_for(const hill_desc* d, int mode, int max_k, int sms) {
                     ? 1
                     : score_deal_warps(d->num_kv_heads, d->num_q_heads / d->num_kv_heads);
   L.attn_grid = sms;
-  L.splits = attn_max_segments(max_k < 0 ? 0 : max_k);
+  L.splits = score_only ? 0 : attn_max_segments(max_k < 0 ? 0 : max_k);
   size_t off = 0;
+  // the step's scores when the caller passes none
   L.scores = off;
-  off += align_up(B * cap * sizeof(float));
+  if (!score_only) off += align_up(B * cap * sizeof(float));
   L.logits = off;
   if (mode == HILL_SCORE_ATTN) off += align_up(B * H * cap * sizeof(float));
   L.partials = off;
@@ -197,7 +201,7 @@ Layout layout_for(const hill_desc* d, int mode, int max_k, int sms) {
   // leading-digit histogram of the selection key, built by the ATTN
   // normalisation when a selection follows (max_k > 0)
   L.hist0 = off;
-  L.has_hist0 = mode == HILL_SCORE_ATTN && max_k > 0;
+  L.has_hist0 = mode == HILL_SCORE_ATTN && max_k > 0 && !score_only;
   if (L.has_hist0) off += align_up(B * (size_t)select_hist_bins() * sizeof(uint32_t));
   L.attn_part = off;
   off += align_up(B * H * (size_t)L.splits * (2 + kHeadDim) * sizeof(float));
@@ -289,7 +293,11 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
     a.nkv = nkv;
     a.hoff = hoff;
     a.Gn = Gn;
-    a.raw_add = first ? 0 : 1;
+    // RAW passes add to what an earlier pass stored in the same rows: every
+    // pass shares the per-sequence rows (b, j), but a per-KV-head row (b, g, j)
+    // is shared only by the query-head passes of KV head g (hoff > 0), so a
+    // later KV-head pass stores into rows no pass has written yet
+    a.raw_add = kvh ? (hoff > 0 ? 1 : 0) : (first ? 0 : 1);
     // the dealing kernel exists for the group template 8 (it is chosen for
     // groups of 5 or more heads, whose passes all fit it)
     const bool deal = L.score_spc > 1;
@@ -427,7 +435,7 @@ hill_status hill_score(const hill_desc* desc, const void* q, const void* k_cache
   if (!aligned16(q) || !aligned16(k_cache)) return HILL_ERR_INVALID_ARG;
   DeviceInfo di;
   if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
-  const Layout L = layout_for(desc, mode, 0, di.sms);
+  const Layout L = layout_for(desc, mode, 0, di.sms, true);
   if (!ws || ws_bytes < L.total) return HILL_ERR_WORKSPACE;
   return run_score(desc, q, k_cache, lens, mode, scores, accum, ws_base(ws), L, di,
                    static_cast<cudaStream_t>(stream));
@@ -586,7 +594,7 @@ hill_status hill_score_f8(const hill_desc* desc, const void* q, const uint8_t* k
   if (!aligned16(q) || !aligned16(k8) || !aligned16(kscale)) return HILL_ERR_INVALID_ARG;
   DeviceInfo di;
   if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
-  const Layout L = layout_for(desc, mode, 0, di.sms);
+  const Layout L = layout_for(desc, mode, 0, di.sms, true);
   if (!ws || ws_bytes < L.total) return HILL_ERR_WORKSPACE;
   return run_score(desc, q, k8, lens, mode, scores, accum, ws_base(ws), L, di, static_cast<cudaStream_t>(stream),
                    nullptr, 0, kscale);
@@ -668,7 +676,7 @@ extern "C" hill_status hill_score_noalloc(const hill_desc* desc, const void* q, 
   if (!aligned16(q) || !aligned16(k_cache)) return HILL_ERR_INVALID_ARG;
   DeviceInfo di;
   if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
-  const Layout L = layout_for(desc, mode, 0, di.sms);
+  const Layout L = layout_for(desc, mode, 0, di.sms, true);
   // the array is already 256-byte aligned: the alignment slack is not needed
   if (L.total - kAlign > (size_t)HILL_SCORE_NOALLOC_MAX_SCRATCH) return HILL_ERR_WORKSPACE;
   void* scratch = nullptr;

@@ -49,7 +49,8 @@ def _run(H, q, K, V, lens_t, k, max_k, mode, accum=None):
     Hkv, cap = K.shape[1], K.shape[2]
     desc = H.make_desc(q, K, V)
     ws = H.alloc_workspace(desc, mode, max_k)
-    scores = torch.zeros(B, Hkv, cap, device="cuda")
+    # NaN-filled, so that a row read before any pass wrote it fails the check
+    scores = torch.full((B, Hkv, cap), float("nan"), device="cuda")
     idx = torch.empty(B, Hkv, max_k, dtype=torch.int32, device="cuda")
     cnt = torch.empty(B, Hkv, dtype=torch.int32, device="cuda")
     out = torch.empty(B, Hq, 128, device="cuda")

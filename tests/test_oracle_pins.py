@@ -275,6 +275,40 @@ def test_quantize_rows_bounds(oracle_mod):
         assert np.all(np.abs(dec - y) <= np.maximum(np.abs(y) / 16, 2.0 ** -10) * (1 + 1e-6))
 
 
+@pytest.mark.parametrize("dtype", [torch.float16, torch.bfloat16])
+def test_quantize_rows_matches_torch_float32_steps_and_e4m3_cast(oracle_mod, dtype):
+    """Sec. 4.4's key shadow, row by row, computed here with torch alone: the
+    row maximum |x| in float32, its reciprocal 448 / amax and the products
+    x * (448 / amax) as float32 tensor operations, saturated to +-448, then
+    torch's own cast to float8_e4m3fn; the scale is amax / 448 in float32.
+    The oracle's codes and scales must equal these bit for bit, so a step the
+    oracle and the kernel might share by mistake (a scale of 448 / amax the
+    other way round, rounding the product in double, truncating instead of
+    rounding, a lost sign) fails here."""
+    g = torch.Generator().manual_seed(41)
+    n, d = 600, 128
+    mag = torch.logspace(-5, 4, n)                                 # row magnitudes across the dtypes' range
+    x = (torch.randn(n, d, generator=g) * mag[:, None]).to(dtype)
+    x[7] = 0.0                                                     # an all-zero row
+    x[8] = 0.0
+    x[8, 3] = -2.5                                                 # one negative entry holds the maximum
+    x[9, :] = x[9, :].abs().neg()                                  # every entry negative
+    x[10, ::2] = 0.0
+    codes, scale = oracle_mod.quantize_rows(x)
+    xf = x.float()
+    amax = xf.abs().amax(dim=1)
+    nz = amax > 0
+    r = torch.full_like(amax, 448.0)
+    r[nz] = torch.tensor(448.0, dtype=torch.float32) / amax[nz]
+    y = (xf * r[:, None]).clamp(-448.0, 448.0)
+    ref_codes = y.to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+    ref_codes[~nz.numpy()] = 0
+    ref_scale = torch.where(nz, amax / torch.tensor(448.0, dtype=torch.float32), torch.zeros_like(amax)).numpy()
+    assert np.array_equal(codes, ref_codes), f"{(codes != ref_codes).sum()} codes differ"
+    assert np.array_equal(scale.view(np.uint32), ref_scale.view(np.uint32))
+    assert codes[8, 3] == 0xFE and np.all(codes[9][codes[9] != 0x80] >= 0x80)
+
+
 def test_logits_q8_is_fp64_matmul_of_dequantized(oracle_mod):
     B, H, Hkv, d, cap = 2, 8, 2, 128, 40
     lens = [40, 23]
