@@ -111,6 +111,22 @@ def config(n: int, *, seed: int = 0, **over) -> Workload:
     return dataclasses.replace(w, **over) if over else w
 
 
+SWEEP_BATCHES = (1, 8, 16)
+SWEEP_LENS = (8192, 65536)
+SWEEP_BUDGETS = (0.05, 0.10, 0.20, 0.50)
+
+
+def sweep_point(batch: int, prompt_len: int, budget_frac: float, *, seed: int = 0, **over) -> Workload:
+    """One point of the budget/batch sweep: the Qwen-7B-shaped stack (32
+    layers, 32 heads MHA, head_dim 128, fp16, Zipf(1.1) skew) with `batch`
+    sequences of `prompt_len` tokens, budget floor(budget_frac * len), 128
+    decode steps with cumulative importance.  The point (8, 65536, 0.2) is
+    config(5) itself."""
+    name = f"cfg5-sweep-b{batch}-{prompt_len // 1024}k-k{round(budget_frac * 100)}"
+    return config(5, seed=seed, name=name, batch=batch, prompt_lens=(prompt_len,) * batch,
+                  budget_frac=budget_frac, **over)
+
+
 def _unit(x: torch.Tensor) -> torch.Tensor:
     return x / x.norm(dim=-1, keepdim=True)
 
