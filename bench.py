@@ -47,7 +47,14 @@ from paper_2602_18750_gb300 import inputs  # noqa: E402
 
 METRIC = "cached tokens scored+selected/sec"
 # keyed by --serial
-SCHEDULES = {False: "layer-pipelined (2 streams, Sec. 4.3)", True: "serial (one fused hill_evict_step per layer)"}
+SCHEDULES = {
+    "split": "layer-pipelined (Sec. 4.3): per layer hill_evict_step_begin (K stream) on one stream, "
+             "hill_evict_step_end (normalisation + selection) on a second and the sparse attention on a third, "
+             "overlapping the K stream of the next layers; three rotating evaluation workspaces",
+    "attn-overlap": "layer-pipelined (Sec. 4.3): per layer hill_evict_step without attention on one stream, "
+                    "the sparse attention on a second stream, overlapping the next layer's evaluation",
+    "serial": "serial (one fused hill_evict_step per layer)",
+}
 UNIT = "tokens/s"
 L2_BYTES = 129 * 1024 * 1024
 
@@ -165,6 +172,127 @@ class ClockSampler:
         if note:
             out["note"] = note
         return out
+
+
+# ---------------------------------------------------------------- schedules
+def pipelined_form(f8: bool, mode: int, accumulate: bool, lres: int) -> str:
+    """The layer-pipelined form of a workload.  The E4M3 scoring has no split
+    form; RAW scoring adds to the running importance inside the K stream, so
+    with one resident layer the next layer's stream would race the selection
+    of the previous one on the same running sums."""
+    if f8 or (accumulate and mode == 1 and lres < 2):
+        return "attn-overlap"
+    return "split"
+
+
+# Evaluation workspaces the split schedule rotates: the K stream of layer l
+# may run while the normalisation and selection of layers l - 1 and l - 2 are
+# still in flight (measured: two leave the 128K workload's stream waiting on
+# the selection; four gain nothing over three)
+SPLIT_WORKSPACES = 3
+
+
+def issue_layers(form, L, st, side, att, with_attn, fused, begin, end, attn):
+    """Issue one decode step over L layers on stream st and the helper
+    streams side and att.  fused(l, with_attn, stream, wi), begin(l, stream,
+    wi), end(l, stream, wi) and attn(l, stream, wi) issue the calls of layer l
+    with workspace wi of their stage (evaluation: 0 .. SPLIT_WORKSPACES - 1,
+    attention: 0 or 1)."""
+    if form == "serial":
+        for l in range(L):
+            fused(l, with_attn, st, 0)
+        return
+    fork = torch.cuda.Event()
+    fork.record(st)
+    side.wait_event(fork)
+    helpers = [side]
+    if form == "split":
+        done = [torch.cuda.Event() for _ in range(L)]
+        if with_attn:
+            att.wait_event(fork)
+            helpers.append(att)
+        nw = SPLIT_WORKSPACES
+        for l in range(L):
+            if l >= nw:
+                st.wait_event(done[l - nw])   # workspace l % nw is free again
+            begin(l, st, l % nw)
+            streamed = torch.cuda.Event()
+            streamed.record(st)
+            side.wait_event(streamed)
+            end(l, side, l % nw)
+            done[l].record(side)
+            if with_attn:
+                att.wait_event(done[l])
+                attn(l, att, l % 2)
+    else:
+        for l in range(L):
+            fused(l, False, st, 0)
+            if with_attn:
+                sel = torch.cuda.Event()
+                sel.record(st)
+                side.wait_event(sel)
+                attn(l, side, 0)
+    for h in helpers:
+        join = torch.cuda.Event()
+        join.record(h)
+        st.wait_event(join)
+
+
+def capture_steps(S, stream, issue):
+    """One CUDA graph per decode step t of issue(t, stream)."""
+    graphs = []
+    for t in range(S):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            issue(t, stream)
+        graphs.append(g)
+    return graphs
+
+
+def time_replays(graphs, order, warmup, stream, dev, clocks_of=None):
+    """Replay `warmup` untimed steps, then time exactly the steps of `order`
+    with CUDA events on the launching stream between barrier + synchronize
+    pairs; with clocks_of (a device index) sample the clocks meanwhile.
+    Returns (ms, clock summary or None)."""
+    S = len(graphs)
+    with torch.cuda.stream(stream):
+        for i in range(warmup):
+            graphs[i % S].replay()
+    stream.synchronize()
+    clocks = None
+    if clocks_of is not None:
+        clocks = ClockSampler(smi_device_id(clocks_of))
+        clocks.wait_first()
+    barrier(dev)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    w0 = time.time()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for t in order:
+            graphs[t].replay()
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    w1 = time.time()
+    barrier(dev)
+    info = None
+    if clocks is not None:
+        info = clocks.summary(w0, w1)
+        clocks.stop()
+    return e0.elapsed_time(e1), info
+
+
+def eval_summary(ms, tokens, k_bytes_per_token, layer_steps, world, peak, form):
+    gbs = tokens * k_bytes_per_token / (ms / 1e3) / 1e9
+    return {
+        "what": "evaluation + selection without attention (score + aggregate + select), all layers",
+        "schedule": SCHEDULES[form],
+        "us_per_layer": round(ms * 1e3 / layer_steps, 2),
+        "tokens_per_s": round(world * tokens / (ms / 1e3), 1),
+        "k_stream_gbs": round(gbs, 1),
+        "k_stream_frac_of_measured_hbm": round(gbs / peak, 4),
+        "k_stream_frac_of_8tbs": round(gbs / 8000.0, 4),
+    }
 
 
 # ---------------------------------------------------------------- helpers
@@ -290,167 +418,107 @@ def run_ours(args):
         new_row = lens_all - 1
         torch.cuda.synchronize()
 
-    def evict(t, l, o, st):
+    # The calls of one decode step, per layer l (workspace wi: 0 or 1)
+    def fused(t, l, with_attn, st, wi):
         r = l % lres
         acc = accum[r] if accum is not None else None
+        o = out[l] if with_attn else None
         if f8:
             hill.hill_quantize_k(desc, Kall[r], new_row[t], lens_all[t], 1, k8_all[r], ks_all[r], st)
             hill.hill_evict_step_f8(desc, q_all[t, l], k8_all[r], ks_all[r], Kall[r], Vall[r], lens_all[t], k_all[t],
-                                    max_k, mode, acc, scores[l], idx[l], count[l], o, ws, st)
+                                    max_k, mode, acc, scores[l], idx[l], count[l], o, wss[wi], st)
         elif bkp:
             hill.hill_evict_step_bkp(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], args.bkp_recent,
-                                     max_k, mode, acc, scores[l], idx[l], count[l], hits[r], o, ws, st)
+                                     max_k, mode, acc, scores[l], idx[l], count[l], hits[r], o, wss[wi], st)
         else:
             hill.hill_evict_step(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], max_k, mode, acc,
-                                 scores[l], idx[l], count[l], o, ws, st)
+                                 scores[l], idx[l], count[l], o, wss[wi], st)
 
-    # Layer-pipelined schedule (the APP analogue, Sec. 4.3; the default): the
-    # evaluation and selection of layer l + 1 run on the main stream while the
-    # sparse attention of layer l runs on a side stream after its selection;
-    # the two phases use separate workspaces.  The serial schedule runs one
-    # fused hill_evict_step per layer.  Both are timed; --serial makes the
-    # serial one the headline.
-    side = torch.cuda.Stream(device=dev)
-    ws_attn = hill.alloc_workspace(desc, mode, max_k, dev)
+    def begin(t, l, st, wi):
+        r = l % lres
+        hill.hill_evict_step_begin(desc, q_all[t, l], Kall[r], lens_all[t], max_k, mode,
+                                   accum[r] if accum is not None else None, scores[l], wss[wi], st)
 
-    def issue_step(t, st, serial=args.serial):
-        if serial:
-            for l in range(L):
-                evict(t, l, out[l], st)
-            return
-        fork = torch.cuda.Event()
-        fork.record(st)
-        side.wait_event(fork)
-        for l in range(L):
-            r = l % lres
-            evict(t, l, None, st)                       # evaluation + selection of layer l
-            sel = torch.cuda.Event()
-            sel.record(st)
-            side.wait_event(sel)
-            hill.hill_gather_sparse_attn(desc, q_all[t, l], Kall[r], Vall[r], idx[l], count[l], max_k, out[l],
-                                         ws_attn, side)
-        join = torch.cuda.Event()
-        join.record(side)
-        st.wait_event(join)
+    def end(t, l, st, wi):
+        r = l % lres
+        hill.hill_evict_step_end(desc, lens_all[t], k_all[t], max_k, mode, accum[r] if accum is not None else None,
+                                 scores[l], idx[l], count[l], wss[wi], recent=max(args.bkp_recent, 0),
+                                 hits=hits[r] if bkp else None, stream=st)
+
+    def attn(t, l, st, wi):
+        r = l % lres
+        hill.hill_gather_sparse_attn(desc, q_all[t, l], Kall[r], Vall[r], idx[l], count[l], max_k, out[l], wsa[wi],
+                                     st)
+
+    side, att = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    wss = [ws] + [hill.alloc_workspace(desc, mode, max_k, dev) for _ in range(SPLIT_WORKSPACES - 1)]   # evaluation
+    wsa = [hill.alloc_workspace(desc, mode, max_k, dev) for _ in range(2)]   # attention
+    piped = pipelined_form(f8, mode, w.accumulate, lres)
+    form = "serial" if args.serial else piped
+    other = piped if args.serial else "serial"
+
+    def issue_step(t, st, frm=form, with_attn=True):
+        issue_layers(frm, L, st, side, att, with_attn, lambda l, a_, s_, i_: fused(t, l, a_, s_, i_),
+                     lambda l, s_, i_: begin(t, l, s_, i_), lambda l, s_, i_: end(t, l, s_, i_),
+                     lambda l, s_, i_: attn(t, l, s_, i_))
 
     # eager warm-up of every kernel shape, then one CUDA graph per decode step
     with torch.cuda.stream(stream):
         issue_step(0, stream)
+        issue_step(0, stream, other)
     hill.hill_sync_status(stream)
-    graphs, launches = [], []
-    for t in range(S):
-        g = torch.cuda.CUDAGraph()
-        n0 = hill.hill_kernel_launches()
-        with torch.cuda.graph(g, stream=stream):
-            issue_step(t, stream)
-        launches.append(hill.hill_kernel_launches() - n0)
-        graphs.append(g)
+    n0 = hill.hill_kernel_launches()
+    graphs = capture_steps(S, stream, lambda t, st: issue_step(t, st))
+    launches = (hill.hill_kernel_launches() - n0) // S   # kernels per decode step (the same for every step)
     if accum is not None:
         accum.zero_()
 
     tokens_of = [L * sum(w.lens_at(t)) for t in range(S)]
     order = [(args.warmup + i) % S for i in range(args.steps)]
-
-    with torch.cuda.stream(stream):
-        for i in range(args.warmup):
-            graphs[i % S].replay()
-    stream.synchronize()
-    hill.hill_sync_status(stream)
+    # bytes of the key stream the scoring reads per token: the 16-bit keys, or
+    # with --f8 the E4M3 codes and one float32 scale per row
+    k_bytes_per_token = Hkv * (d + 4) if f8 else Hkv * d * 2
 
     # ---------------- timed region (device-resident inputs)
-    clocks = ClockSampler(smi_device_id(local))
-    clocks.wait_first()
-    barrier(dev)
-    torch.cuda.synchronize(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    w0 = time.time()
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for t in order:
-            graphs[t].replay()
-        e1.record(stream)
-    torch.cuda.synchronize(dev)
-    w1 = time.time()
-    barrier(dev)
-    ms_local = e0.elapsed_time(e1)
-    clock_info = clocks.summary(w0, w1)
-    clocks.stop()
+    ms_local, clock_info = time_replays(graphs, order, args.warmup, stream, dev, clocks_of=local)
     hill.hill_sync_status(stream)
     ms = max_over_ranks(ms_local, dev)
     tokens = sum(tokens_of[t] for t in order)
     value = world * tokens / (ms / 1e3)
-    # bytes of the key stream the scoring reads per token: the 16-bit keys, or
-    # with --f8 the E4M3 codes and one float32 scale per row
-    k_bytes_per_token = Hkv * (d + 4) if f8 else Hkv * d * 2
     k_gbs = world * tokens * k_bytes_per_token / (ms / 1e3) / 1e9
-    gpu_launches = sum(launches[t] for t in order)
+    gpu_launches = launches * len(order)
+    del graphs
 
     # ---------------- the other schedule, the same steps, timed the same way
-    other_graphs = []
-    for t in range(S):
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            issue_step(t, stream, serial=not args.serial)
-        other_graphs.append(g)
     if accum is not None:
         accum.zero_()
-    with torch.cuda.stream(stream):
-        for i in range(args.warmup):
-            other_graphs[i % S].replay()
-    barrier(dev)
-    torch.cuda.synchronize(dev)
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for t in order:
-            other_graphs[t].replay()
-        e1.record(stream)
-    torch.cuda.synchronize(dev)
-    barrier(dev)
-    ms_other = max_over_ranks(e0.elapsed_time(e1), dev)
+    other_graphs = capture_steps(S, stream, lambda t, st: issue_step(t, st, other))
+    ms_other = max_over_ranks(time_replays(other_graphs, order, args.warmup, stream, dev)[0], dev)
     hill.hill_sync_status(stream)
     other_schedule = {
-        "schedule": SCHEDULES[not args.serial],
+        "schedule": SCHEDULES[other],
         "us_per_layer": round(ms_other * 1e3 / (len(order) * L), 2),
         "tokens_per_s": round(world * tokens / (ms_other / 1e3), 1),
     }
     del other_graphs
 
     # ---------------- evaluation + selection only (no attention): the same steps
-    # with out = NULL, one graph per decode step, timed like the main region
-    def issue_eval(t, st):
-        for l in range(L):
-            evict(t, l, None, st)
-
-    eval_graphs = []
-    for t in range(S):
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            issue_eval(t, stream)
-        eval_graphs.append(g)
-    with torch.cuda.stream(stream):
-        for i in range(args.warmup):
-            eval_graphs[i % S].replay()
-    barrier(dev)
-    torch.cuda.synchronize(dev)
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for t in order:
-            eval_graphs[t].replay()
-        e1.record(stream)
-    torch.cuda.synchronize(dev)
-    barrier(dev)
-    ms_eval = max_over_ranks(e0.elapsed_time(e1), dev)
-    hill.hill_sync_status(stream)
-    eval_gbs = tokens * k_bytes_per_token / (ms_eval / 1e3) / 1e9
+    # with out = NULL, in the pipelined form (the K stream of layer l + 1
+    # overlaps the normalisation and selection of layer l) and serially, one
+    # graph per decode step, timed like the main region
     peak, peak_kind = measured_peaks()
-    eval_select = {
-        "what": "hill_evict_step without attention (score + aggregate + select), all layers",
-        "us_per_layer": round(ms_eval * 1e3 / (len(order) * L), 2),
-        "tokens_per_s": round(world * tokens / (ms_eval / 1e3), 1),
-        "k_stream_gbs": round(eval_gbs, 1),
-        "k_stream_frac_of_measured_hbm": round(eval_gbs / peak, 4),
-        "k_stream_frac_of_8tbs": round(eval_gbs / 8000.0, 4),
-    }
+    eval_forms = {}
+    for frm in dict.fromkeys([piped, "serial"]):
+        if accum is not None:
+            accum.zero_()
+        eg = capture_steps(S, stream, lambda t, st: issue_step(t, st, frm, with_attn=False))
+        ms_e = max_over_ranks(time_replays(eg, order, args.warmup, stream, dev)[0], dev)
+        hill.hill_sync_status(stream)
+        del eg
+        eval_forms[frm] = eval_summary(ms_e, tokens, k_bytes_per_token, len(order) * L, world, peak, frm)
+    eval_select = dict(eval_forms[piped])
+    if piped != "serial":
+        eval_select["serial"] = eval_forms["serial"]
 
     # ---------------- scoring stage alone, per launch (roofline of the dominant kernels)
     t_s = S - 1
@@ -494,7 +562,7 @@ def run_ours(args):
     e2e = None
     if not args.no_e2e:
         e2e = run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all, accum, scores,
-                      idx, count, out, ws, stream, dev, world, side, ws_attn)
+                      idx, count, out, wss, wsa, stream, dev, world, side, att, form)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -509,8 +577,7 @@ def run_ours(args):
         acceptance = {"target": "evaluation + selection K stream >= 0.70 of 8 TB/s at >= 32K tokens"}
         if w.name == inputs.config(3).name:
             acceptance["cfg3"] = dict(eval_select, workload=w.name)
-        del graphs, eval_graphs
-        del Kall, Vall, q_all, accum, scores, idx, count, out, ws, ws_attn
+        del Kall, Vall, q_all, accum, scores, idx, count, out, ws, wss, wsa
         torch.cuda.empty_cache()
         for n in (3, 4):
             name = inputs.config(n).name
@@ -525,7 +592,7 @@ def run_ours(args):
             "data": "synthetic", "config": dict(describe(w, lres, args.mode),
                                                 **({"bkp_recent": args.bkp_recent} if bkp else {}),
                                                 **({"scoring": "e4m3 key shadow"} if f8 else {}),
-                                                schedule=SCHEDULES[args.serial]),
+                                                schedule=SCHEDULES[form]),
             "k_stream_gbs": round(k_gbs, 1),
             "k_stream_frac_of_measured_hbm": round(k_gbs / world / peak, 4),
             "k_stream_frac_of_8tbs": round(k_gbs / world / 8000.0, 4),
@@ -542,13 +609,13 @@ def run_ours(args):
 
 
 def eval_select_only(args, n, hill, dev, world, mode):
-    """Evaluation + selection alone (hill_evict_step without attention, one
-    CUDA graph per decode step over all layers) on workload n, with all its
-    layers resident, timed like the main region; plus the scoring stage
-    (hill_score) per launch.  Used for the contexts of 32K tokens or more that
-    the headline workload does not cover."""
+    """Evaluation + selection alone (no attention) on workload n with all its
+    layers resident (as many as fit), in the layer-pipelined form and
+    serially, one CUDA graph per decode step over all layers, timed like the
+    main region; plus the scoring stage (hill_score) per launch.  Used for the
+    contexts of 32K tokens or more that the headline workload does not cover."""
     rank, _, local = dist_env()
-    w, lres = workload_for(n, replica_seed(args.seed, rank), None)
+    w, _ = workload_for(n, replica_seed(args.seed, rank), None)
     L, S, B, Hq, Hkv, d = w.layers, w.steps, w.batch, w.heads, w.kv_heads, w.head_dim
     per_layer = 2 * B * Hkv * w.capacity * d * torch.finfo(w.dtype).bits // 8
     lres = max(1, min(L, int(0.7 * torch.cuda.mem_get_info(dev)[0]) // per_layer))
@@ -567,52 +634,45 @@ def eval_select_only(args, n, hill, dev, world, mode):
     idx = torch.empty(L, B, w.max_k, dtype=torch.int32, device=dev)
     count = torch.empty(L, B, dtype=torch.int32, device=dev)
     desc = hill.make_desc(q_all[0, 0], Kall[0], Vall[0])
-    ws = hill.alloc_workspace(desc, mode, w.max_k, dev)
-    stream = torch.cuda.Stream(device=dev)
+    wss = [hill.alloc_workspace(desc, mode, w.max_k, dev) for _ in range(SPLIT_WORKSPACES)]
+    stream, side = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    torch.cuda.synchronize(dev)   # the inputs were made on the default stream
 
-    def issue(t):
-        for l in range(L):
-            r = l % lres
-            hill.hill_evict_step(desc, q_all[t, l], Kall[r], Vall[r], lens_all[t], k_all[t], w.max_k, mode,
-                                 accum[r] if accum is not None else None, scores[l], idx[l], count[l], None, ws,
-                                 stream)
+    def acc(l):
+        return accum[l % lres] if accum is not None else None
 
-    with torch.cuda.stream(stream):
-        issue(0)
-    hill.hill_sync_status(stream)
-    graphs = []
-    for t in range(S):
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            issue(t)
-        graphs.append(g)
-    if accum is not None:
-        accum.zero_()
+    def issue(t, st, frm):
+        def fused(l, _, s_, wi):
+            hill.hill_evict_step(desc, q_all[t, l], Kall[l % lres], Vall[l % lres], lens_all[t], k_all[t], w.max_k,
+                                 mode, acc(l), scores[l], idx[l], count[l], None, wss[wi], s_)
+
+        def begin(l, s_, wi):
+            hill.hill_evict_step_begin(desc, q_all[t, l], Kall[l % lres], lens_all[t], w.max_k, mode, acc(l),
+                                       scores[l], wss[wi], s_)
+
+        def end(l, s_, wi):
+            hill.hill_evict_step_end(desc, lens_all[t], k_all[t], w.max_k, mode, acc(l), scores[l], idx[l],
+                                     count[l], wss[wi], stream=s_)
+
+        issue_layers(frm, L, st, side, None, False, fused, begin, end, None)
+
     order = [(args.warmup + i) % S for i in range(args.steps)]
-    with torch.cuda.stream(stream):
-        for i in range(args.warmup):
-            graphs[i % S].replay()
-    stream.synchronize()
-    clocks = ClockSampler(smi_device_id(local))
-    clocks.wait_first()
-    barrier(dev)
-    torch.cuda.synchronize(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    w0 = time.time()
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for t in order:
-            graphs[t].replay()
-        e1.record(stream)
-    torch.cuda.synchronize(dev)
-    w1 = time.time()
-    barrier(dev)
-    clock_info = clocks.summary(w0, w1)
-    clocks.stop()
-    ms = max_over_ranks(e0.elapsed_time(e1), dev)
-    hill.hill_sync_status(stream)
     tokens = sum(L * sum(w.lens_at(t)) for t in order)
-    gbs = tokens * Hkv * d * 2 / (ms / 1e3) / 1e9
+    peak, _ = measured_peaks()
+    piped = pipelined_form(False, mode, w.accumulate, lres)
+    forms = {}
+    for frm in dict.fromkeys([piped, "serial"]):
+        with torch.cuda.stream(stream):
+            issue(0, stream, frm)
+        hill.hill_sync_status(stream)
+        graphs = capture_steps(S, stream, lambda t, st: issue(t, st, frm))
+        if accum is not None:
+            accum.zero_()
+        ms, clock_info = time_replays(graphs, order, args.warmup, stream, dev, clocks_of=local)
+        ms = max_over_ranks(ms, dev)
+        hill.hill_sync_status(stream)
+        del graphs
+        forms[frm] = dict(eval_summary(ms, tokens, Hkv * d * 2, len(order) * L, world, peak, frm), clocks=clock_info)
     # the scoring stage alone, per launch, at the last decode step
     t_s = S - 1
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(L)]
@@ -622,38 +682,33 @@ def eval_select_only(args, n, hill, dev, world, mode):
             for l in range(L):
                 if rep == 1:
                     starts[l].record(stream)
-                hill.hill_score(desc, q_all[t_s, l], Kall[l % lres], lens_all[t_s], mode, scores[l], None, ws, stream)
+                hill.hill_score(desc, q_all[t_s, l], Kall[l % lres], lens_all[t_s], mode, scores[l], None, wss[0],
+                                stream)
                 if rep == 1:
                     ends[l].record(stream)
     stream.synchronize()
     hill.hill_sync_status(stream)
     score_us = sum(a.elapsed_time(b) for a, b in zip(starts, ends)) / L * 1e3
-    peak, _ = measured_peaks()
-    out = {
+    out = dict(forms[piped])
+    if piped != "serial":
+        out["serial"] = forms["serial"]
+    out.update({
         "workload": w.name, "batch": B, "heads": Hq, "kv_heads": Hkv, "kv_dtype": str(w.dtype).replace("torch.", ""),
         "tokens_last_step": w.lens_at(S - 1), "layers_resident": lres, "steps_timed": len(order),
-        "what": "hill_evict_step without attention (score + aggregate + select), all layers",
-        "us_per_layer": round(ms * 1e3 / (len(order) * L), 2),
-        "tokens_per_s": round(world * tokens / (ms / 1e3), 1),
-        "k_stream_gbs": round(gbs, 1),
-        "k_stream_frac_of_measured_hbm": round(gbs / peak, 4),
-        "k_stream_frac_of_8tbs": round(gbs / 8000.0, 4),
         "scoring_stage_us": round(score_us, 2),
         "scoring_stage_frac_of_measured_hbm": round(
             sum(w.lens_at(t_s)) * (Hkv * d * 2 + 4) / (score_us / 1e6) / 1e9 / peak, 4),
-        "clocks": clock_info,
-    }
-    del graphs, Kall, Vall, q_all, accum, scores, idx, count, ws
+    })
+    del Kall, Vall, q_all, accum, scores, idx, count, wss
     torch.cuda.empty_cache()
     return out
 
 
 def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all, accum, scores, idx, count,
-            out, ws, stream, dev, world, side, ws_attn):
-    """Same steps through the public calls (eager, in the bench's schedule:
-    hill_evict_step per layer, or with the layer-pipelined schedule
-    hill_evict_step without attention on the main stream and
-    hill_gather_sparse_attn on the side stream), with each step's inputs
+            out, wss, wsa, stream, dev, world, side, att, form):
+    """Same steps through the public calls, in the bench's schedule (one
+    fused hill_evict_step per layer, or the layer-pipelined begin / end plus
+    hill_gather_sparse_attn on a second stream), with each step's inputs
     copied from pinned host memory (query of every layer, the new token's K/V
     row of every layer, lengths, budgets) and its results (selection and
     attention output of every layer) copied back, all inside the timed region."""
@@ -677,42 +732,52 @@ def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all,
     cnt_h = torch.empty_like(count, device="cpu").pin_memory()
     out_h = torch.empty_like(out, device="cpu").pin_memory()
     uniform = [len(set(p)) == 1 for p in pos]
-    # per-layer views and events, made once (as an engine would hold them)
+    # per-layer views, made once (as an engine would hold them)
     qv = [[q_all[t, l] for l in range(L)] for t in range(S)]
     Kv, Vv = [Kall[r] for r in range(lres)], [Vall[r] for r in range(lres)]
     accv = [accum[r] if accum is not None else None for r in range(lres)]
-    idxv, cntv, outv, scv = list(idx), list(count), list(out), list(scores)
-    lens_d, kk_d = lk_d[0], lk_d[1]
-    fork, join = torch.cuda.Event(), torch.cuda.Event()
-    sel = [torch.cuda.Event() for _ in range(L)]
+    scv = list(scores)
+
+    def compute(t, lens_d, kk_d, ri, rc, ro):
+        """The step's calls on the device buffers: lengths/budgets lens_d,
+        kk_d; results into the per-layer views ri, rc, ro."""
+        def fused(l, with_attn, st, wi):
+            r = l % lres
+            hill.hill_evict_step(desc, qv[t][l], Kv[r], Vv[r], lens_d, kk_d, w.max_k, mode, accv[r], scv[l], ri[l],
+                                 rc[l], ro[l] if with_attn else None, wss[wi], st)
+
+        def begin(l, st, wi):
+            hill.hill_evict_step_begin(desc, qv[t][l], Kv[l % lres], lens_d, w.max_k, mode, accv[l % lres], scv[l],
+                                       wss[wi], st)
+
+        def end(l, st, wi):
+            hill.hill_evict_step_end(desc, lens_d, kk_d, w.max_k, mode, accv[l % lres], scv[l], ri[l], rc[l],
+                                     wss[wi], stream=st)
+
+        def attn(l, st, wi):
+            r = l % lres
+            hill.hill_gather_sparse_attn(desc, qv[t][l], Kv[r], Vv[r], ri[l], rc[l], w.max_k, ro[l], wsa[wi], st)
+
+        issue_layers(form, L, stream, side, att, True, fused, begin, end, attn)
+
+    def append(t, sk, sv):
+        if uniform[t]:
+            Kall[:, :, :, pos[t][0]].copy_(sk)
+            Vall[:, :, :, pos[t][0]].copy_(sv)
+        else:
+            for b in range(B):
+                Kall[:, b, :, pos[t][b]].copy_(sk[:, b])
+                Vall[:, b, :, pos[t][b]].copy_(sv[:, b])
+
+    res0 = (list(idx), list(count), list(out))
 
     def one(t):
         q_all[t].copy_(q_h[t], non_blocking=True)
         stage_k.copy_(newk_h[t], non_blocking=True)
         stage_v.copy_(newv_h[t], non_blocking=True)
         lk_d.copy_(lk_h[t], non_blocking=True)
-        if uniform[t]:
-            Kall[:, :, :, pos[t][0]].copy_(stage_k)
-            Vall[:, :, :, pos[t][0]].copy_(stage_v)
-        else:
-            for b in range(B):
-                Kall[:, b, :, pos[t][b]].copy_(stage_k[:, b])
-                Vall[:, b, :, pos[t][b]].copy_(stage_v[:, b])
-        if not args.serial:
-            fork.record(stream)
-            side.wait_event(fork)
-        for l in range(L):
-            r = l % lres
-            hill.hill_evict_step(desc, qv[t][l], Kv[r], Vv[r], lens_d, kk_d, w.max_k, mode, accv[r], scv[l],
-                                 idxv[l], cntv[l], outv[l] if args.serial else None, ws, stream)
-            if not args.serial:
-                sel[l].record(stream)
-                side.wait_event(sel[l])
-                hill.hill_gather_sparse_attn(desc, qv[t][l], Kv[r], Vv[r], idxv[l], cntv[l], w.max_k, outv[l],
-                                             ws_attn, side)
-        if not args.serial:
-            join.record(side)
-            stream.wait_event(join)
+        append(t, stage_k, stage_v)
+        compute(t, lk_d[0], lk_d[1], *res0)
         idx_h.copy_(idx, non_blocking=True)
         cnt_h.copy_(count, non_blocking=True)
         out_h.copy_(out, non_blocking=True)
@@ -745,31 +810,8 @@ def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all,
             cnt_h.copy_(pc, non_blocking=True)
             out_h.copy_(po, non_blocking=True)
         cjoin.record(cstream)
-        sk, sv = stage2_k[par], stage2_v[par]
-        if uniform[t]:
-            Kall[:, :, :, pos[t][0]].copy_(sk)
-            Vall[:, :, :, pos[t][0]].copy_(sv)
-        else:
-            for b in range(B):
-                Kall[:, b, :, pos[t][b]].copy_(sk[:, b])
-                Vall[:, b, :, pos[t][b]].copy_(sv[:, b])
-        ld, kd = lk2_d[par][0], lk2_d[par][1]
-        ri, rc, ro = resv[par]
-        if not args.serial:
-            fork.record(stream)
-            side.wait_event(fork)
-        for l in range(L):
-            r = l % lres
-            hill.hill_evict_step(desc, qv[t][l], Kv[r], Vv[r], ld, kd, w.max_k, mode, accv[r], scv[l], ri[l],
-                                 rc[l], ro[l] if args.serial else None, ws, stream)
-            if not args.serial:
-                sel[l].record(stream)
-                side.wait_event(sel[l])
-                hill.hill_gather_sparse_attn(desc, qv[t][l], Kv[r], Vv[r], ri[l], rc[l], w.max_k, ro[l],
-                                             ws_attn, side)
-        if not args.serial:
-            join.record(side)
-            stream.wait_event(join)
+        append(t, stage2_k[par], stage2_v[par])
+        compute(t, lk2_d[par][0], lk2_d[par][1], *resv[par])
         stream.wait_event(cjoin)
 
     def timed(step_fn):
@@ -821,17 +863,16 @@ def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all,
     h2d = (q_h[0].numel() * q_h.element_size() + 2 * newk_h[0].numel() * newk_h.element_size()
            + lk_h[0].numel() * 4)
     d2h = idx_h.numel() * 4 + cnt_h.numel() * 4 + out_h.numel() * 4
-    calls = ("hill_evict_step per layer" if args.serial else
-             "hill_evict_step (no attention) + hill_gather_sparse_attn on a second stream, per layer")
+    calls = SCHEDULES[form]
     return {"value": round(world * tokens / (ms / 1e3), 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": round(ms / len(order), 4),
-            "api": calls + ", captured per decode step in a CUDA graph and replayed; every step copies one "
+            "api": calls + "; captured per decode step in a CUDA graph and replayed; every step copies one "
                            "step's inputs in from pinned host memory and one step's results out to pinned host "
                            "memory on a copy stream, overlapped with the compute (next step's inputs, previous "
                            "step's results; two alternating buffer sets)",
             "eager": {"value": round(world * tokens / (ms_eager / 1e3), 1),
                       "ms_per_step": round(ms_eager / len(order), 4),
-                      "api": calls + ", issued from Python at every step (no graph)"}}
+                      "api": calls + "; issued from Python at every step (no graph)"}}
 
 
 def cpu_baseline(w, lres, Kall, Vall, q_all, mode, seconds=10.0):

@@ -168,6 +168,45 @@ hill_status hill_evict_step_bkp(const hill_desc* desc, const void* q, const void
                                 float* scores, int32_t* idx, int32_t* count, uint16_t* hits, float* out,
                                 void* ws, size_t ws_bytes, void* stream);
 
+/* The same step in two calls, for the layer-pipelined evaluation of Sec. 4.3
+ * (the evaluation of layer i + 1 overlaps the rest of layer i): while the
+ * normalisation and selection of one layer run on a second stream, the K
+ * stream of the next layer proceeds on the first.
+ *
+ * hill_evict_step_begin launches the scoring kernel: it streams the K cache
+ * once and writes, in ATTN mode, the logits and per-CTA softmax partials into
+ * the workspace, in RAW mode the per-token sums into scores (and accum +=).
+ * It reads q, k_cache and lens.
+ *
+ * hill_evict_step_end completes the step from the workspace: in ATTN mode the
+ * normalisation (scores, accum += as in hill_score), then the top-k selection
+ * of hill_topk_select_bkp (recent = 0 and hits = NULL: exactly
+ * hill_topk_select) on accum if given, else on this step's scores.  It reads
+ * no keys.  Its kernels are sized to share the GPU's multiprocessors with a
+ * scoring kernel running at the same time (the selection runs as clusters of
+ * at most 8 CTAs of 256 threads per sequence, re-reading the keys from
+ * global memory).
+ *
+ * Both calls of one step take the same desc, lens, max_k, mode, accum,
+ * scores and ws (sized by hill_workspace_bytes); end may be issued on another
+ * stream than begin, after an event recorded behind begin.  The workspace
+ * belongs to the step from begin until end has completed: a pipeline over
+ * layers rotates n >= 2 workspaces and issues begin of layer l + n only after
+ * end of layer l (three let the K stream run two layers ahead of the
+ * selection).  The scoring kernel of begin takes four fifths of the SMs, so
+ * that end's kernels have room beside it.  Results equal those of
+ * hill_evict_step_bkp without attention (scores within rounding: the split
+ * normalisation always combines the softmax partials in a kernel of its own;
+ * selections follow the same rule).  Attention: hill_gather_sparse_attn on idx
+ * and count afterwards. */
+hill_status hill_evict_step_begin(const hill_desc* desc, const void* q, const void* k_cache,
+                                  const int32_t* lens, int32_t max_k, hill_score_mode mode, float* accum,
+                                  float* scores, void* ws, size_t ws_bytes, void* stream);
+hill_status hill_evict_step_end(const hill_desc* desc, const int32_t* lens, const int32_t* k, int32_t recent,
+                                int32_t max_k, hill_score_mode mode, float* accum, float* scores,
+                                int32_t* idx, int32_t* count, uint16_t* hits, void* ws, size_t ws_bytes,
+                                void* stream);
+
 /* Per-KV-head selection (a variant of the evaluation: the paper evaluates at
  * token level for every head topology, Sec. 5.3; here each KV head keeps its
  * own set).  The importance is aggregated over the G query heads of each KV

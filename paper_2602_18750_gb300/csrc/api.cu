@@ -164,10 +164,14 @@ struct Layout {
   int score_spc;   // ATTN partial slots per scoring CTA
 };
 
-int score_grid_for(const hill_desc* d, int sms) {
+// The scoring kernel's grid: one CTA per SM, or in the split step
+// (split_grid) four fifths of them, so that the normalisation and selection of
+// the previous layer find whole SMs beside the K stream (the stream itself is
+// bound by HBM, not by the number of SMs streaming).
+int score_grid_for(const hill_desc* d, int sms, bool split_grid = false) {
   const int T = score_tile_tokens();
   const long long items = (long long)d->batch * ((d->capacity + T - 1) / T);
-  long long g = sms;
+  long long g = split_grid ? sms * 4 / 5 : sms;
   if (items < g) g = items;
   return g < 1 ? 1 : (int)g;
 }
@@ -175,10 +179,11 @@ int score_grid_for(const hill_desc* d, int sms) {
 // Workspace regions of a call.  score_only: hill_score and its variants,
 // which write the caller's scores and run no selection or attention, need
 // only the ATTN normalisation's logits, partials and statistics.
-Layout layout_for(const hill_desc* d, int mode, int max_k, int sms, bool score_only = false) {
+Layout layout_for(const hill_desc* d, int mode, int max_k, int sms, bool score_only = false,
+                  bool split_grid = false) {
   Layout L{};
   const size_t B = d->batch, H = d->num_q_heads, cap = d->capacity;
-  L.score_grid = score_grid_for(d, sms);
+  L.score_grid = score_grid_for(d, sms, split_grid);
   // few KV heads with large groups (MQA-like): the scoring kernel deals the
   // tiles to several warps per head, each with its own partial slot (more
   // than score_max_kv_heads() KV heads run in passes of at least half that)
@@ -191,8 +196,9 @@ Layout layout_for(const hill_desc* d, int mode, int max_k, int sms, bool score_o
   // the step's scores when the caller passes none
   L.scores = off;
   if (!score_only) off += align_up(B * cap * sizeof(float));
+  // logits, rows padded to 32 tokens (one 128-byte line per warp and head)
   L.logits = off;
-  if (mode == HILL_SCORE_ATTN) off += align_up(B * H * cap * sizeof(float));
+  if (mode == HILL_SCORE_ATTN) off += align_up(B * H * (size_t)cap32_of(d) * sizeof(float));
   L.partials = off;
   if (mode == HILL_SCORE_ATTN) off += align_up(B * (size_t)L.score_grid * L.score_spc * H * sizeof(float2));
   // combined (max, 1/sum) per (b, h), when the normalisation runs in two kernels
@@ -245,10 +251,14 @@ hill_status head_passes(const hill_desc* d, bool kv_split, F&& f) {
   return HILL_OK;
 }
 
+// Which part of the scoring stage run_score launches: all of it, the K
+// stream only (the scoring kernel), or the ATTN normalisation only.
+constexpr int kScoreAll = 0, kScoreStream = 1, kScoreNormalise = 2;
+
 hill_status run_score(const hill_desc* d, const void* q, const void* k, const int32_t* lens, int mode,
                       float* scores, float* accum, unsigned char* base, const Layout& L,
                       const DeviceInfo& di, cudaStream_t st, uint32_t* hist0 = nullptr, int recent = 0,
-                      const float* kscale = nullptr, bool kvh = false) {
+                      const float* kscale = nullptr, bool kvh = false, int part = kScoreAll) {
   if (d->batch == 0 || d->capacity == 0) return HILL_OK;
   const int G = d->num_q_heads / d->num_kv_heads;
   ScoreArgs a{};
@@ -268,8 +278,10 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   a.err = di.err;
   // kscale != NULL: k is the E4M3 shadow of the keys (asymmetric-precision scoring)
   const bool f8 = kscale != nullptr;
-  hill_status ms = f8 ? make_kmap8(d, k, &a) : make_kmap(d, k, &a);
-  if (ms != HILL_OK) return ms;
+  if (part != kScoreNormalise) {   // the normalisation alone reads no keys
+    const hill_status ms = f8 ? make_kmap8(d, k, &a) : make_kmap(d, k, &a);
+    if (ms != HILL_OK) return ms;
+  }
   a.kscale = kscale;
   a.cap32 = cap32_of(d);
   const bool raw = mode == HILL_SCORE_RAW;
@@ -279,6 +291,7 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
     a.accum = accum;
   } else {
     a.logits = reinterpret_cast<float*>(base + L.logits);
+    a.lstride = cap32_of(d);
     a.partials = reinterpret_cast<float2*>(base + L.partials);
     a.hist0 = hist0;
     a.hist0_words = (int64_t)d->batch * select_hist_bins();
@@ -288,7 +301,8 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   // own keys (RAW passes after the first add their sums); the kernel's group
   // template is the power of two at or above the pass's heads
   a.Gs = G;
-  hill_status s = head_passes(d, true, [&](int goff, int nkv, int hoff, int Gn, bool first) {
+  hill_status s = part == kScoreNormalise ? HILL_OK : head_passes(d, true, [&](int goff, int nkv, int hoff, int Gn,
+                                                                                bool first) {
     a.goff = goff;
     a.nkv = nkv;
     a.hoff = hoff;
@@ -304,9 +318,10 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
     return from_cuda(
         counted(launch_score(a, d->dtype, deal ? 8 : pow2_at_least(Gn), raw, f8, deal, L.score_grid, st), 1));
   });
-  if (s != HILL_OK || raw) return s;
+  if (s != HILL_OK || raw || part == kScoreStream) return s;
   FinalizeArgs f{};
   f.logits = a.logits;
+  f.lstride = a.lstride;
   f.partials = a.partials;
   f.lens = lens;
   f.B = d->batch;
@@ -322,14 +337,16 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   f.Hkv = d->num_kv_heads;
   f.stats = reinterpret_cast<float2*>(base + L.stats);
   int kernels = 0;
-  const cudaError_t e = launch_attn_finalize(f, di.sms, st, &kernels);
+  // the split step's normalisation takes the two-kernel form, whose finalize
+  // kernel fits beside a scoring CTA on one SM
+  const cudaError_t e = launch_attn_finalize(f, di.sms, st, &kernels, part == kScoreNormalise);
   return from_cuda(counted(e, kernels));
 }
 
 hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens, const int32_t* k,
                        int max_k, int32_t* idx, int32_t* count, const DeviceInfo& di, cudaStream_t st,
                        const uint32_t* hist0 = nullptr, int recent = 0, uint16_t* hits = nullptr,
-                       bool kvh = false) {
+                       bool kvh = false, bool lean = false) {
   if (d->batch == 0) return HILL_OK;
   SelectArgs a{};
   a.key = key;
@@ -345,7 +362,7 @@ hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens
   a.hits = hits;
   a.rows_per_seq = kvh ? d->num_kv_heads : 1;
   a.err = di.err;
-  return from_cuda(counted(launch_select(a, st), 1));
+  return from_cuda(counted(lean ? launch_select_lean(a, st) : launch_select(a, st), 1));
 }
 
 hill_status run_attn(const hill_desc* d, const void* q, const void* k, const void* v, const int32_t* idx,
@@ -530,6 +547,49 @@ hill_status hill_topk_select_bkp(const hill_desc* desc, const float* scores, con
   if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
   return run_select(desc, scores, lens, k, max_k, idx, count, di, static_cast<cudaStream_t>(stream), nullptr,
                     recent, hits);
+}
+
+hill_status hill_evict_step_begin(const hill_desc* desc, const void* q, const void* k_cache, const int32_t* lens,
+                                  int32_t max_k, hill_score_mode mode, float* accum, float* scores, void* ws,
+                                  size_t ws_bytes, void* stream) {
+  hill_status s = check_desc(desc);
+  if (s != HILL_OK) return s;
+  if (mode != HILL_SCORE_ATTN && mode != HILL_SCORE_RAW) return HILL_ERR_INVALID_ARG;
+  if (max_k < 0 || !q || !k_cache || !lens) return HILL_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k_cache)) return HILL_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  const Layout L = layout_for(desc, mode, max_k, di.sms, false, true);
+  if (!ws || ws_bytes < L.total) return HILL_ERR_WORKSPACE;
+  unsigned char* base = ws_base(ws);
+  float* s_out = scores ? scores : (accum ? nullptr : reinterpret_cast<float*>(base + L.scores));
+  uint32_t* hist0 = L.has_hist0 ? reinterpret_cast<uint32_t*>(base + L.hist0) : nullptr;
+  return run_score(desc, q, k_cache, lens, mode, s_out, accum, base, L, di, static_cast<cudaStream_t>(stream),
+                   hist0, 0, nullptr, false, kScoreStream);
+}
+
+hill_status hill_evict_step_end(const hill_desc* desc, const int32_t* lens, const int32_t* k, int32_t recent,
+                                int32_t max_k, hill_score_mode mode, float* accum, float* scores, int32_t* idx,
+                                int32_t* count, uint16_t* hits, void* ws, size_t ws_bytes, void* stream) {
+  hill_status s = check_desc(desc);
+  if (s != HILL_OK) return s;
+  if (mode != HILL_SCORE_ATTN && mode != HILL_SCORE_RAW) return HILL_ERR_INVALID_ARG;
+  if (max_k < 0 || recent < 0 || !lens || !k || !count || (max_k > 0 && !idx)) return HILL_ERR_INVALID_ARG;
+  DeviceInfo di;
+  if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
+  const Layout L = layout_for(desc, mode, max_k, di.sms, false, true);
+  if (!ws || ws_bytes < L.total) return HILL_ERR_WORKSPACE;
+  unsigned char* base = ws_base(ws);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  float* s_out = scores ? scores : (accum ? nullptr : reinterpret_cast<float*>(base + L.scores));
+  uint32_t* hist0 = L.has_hist0 ? reinterpret_cast<uint32_t*>(base + L.hist0) : nullptr;
+  if (mode == HILL_SCORE_ATTN) {
+    s = run_score(desc, nullptr, nullptr, lens, mode, s_out, accum, base, L, di, st, hist0, recent, nullptr, false,
+                  kScoreNormalise);
+    if (s != HILL_OK) return s;
+  }
+  return run_select(desc, accum ? accum : s_out, lens, k, max_k, idx, count, di, st, hist0, recent, hits, false,
+                    true);
 }
 
 hill_status hill_evict_step_kvh(const hill_desc* desc, const void* q, const void* k_cache, const void* v_cache,

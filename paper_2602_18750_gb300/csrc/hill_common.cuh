@@ -120,6 +120,20 @@ __device__ __forceinline__ uint64_t l2_evict_first_policy() {
   return pol;
 }
 
+// L2 policy for scratch data written now and read back soon (the ATTN
+// logits): kept in L2 ahead of the streamed keys until it is read and
+// discarded.
+__device__ __forceinline__ uint64_t l2_evict_last_policy() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+// 32-bit global store with an L2 cache-policy hint.
+__device__ __forceinline__ void st_global_hint(float* p, float v, uint64_t policy) {
+  asm volatile("st.global.L2::cache_hint.f32 [%0], %1, %2;" ::"l"(p), "f"(v), "l"(policy) : "memory");
+}
+
 // Bulk (non-tensor) TMA copy global -> this CTA's shared memory, completing
 // `bytes` of transaction count on `bar`.  Addresses and size: multiples of 16.
 __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar,
@@ -164,6 +178,12 @@ __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// Invalidate the 128-byte L2 line at p (128-byte aligned) without writing it
+// back: for scratch data that no one reads again.
+__device__ __forceinline__ void l2_discard_line(const void* p) {
+  asm volatile("discard.global.L2 [%0], 128;" ::"l"(p) : "memory");
 }
 
 __device__ __forceinline__ void prefetch_tmap(const void* tmap) {

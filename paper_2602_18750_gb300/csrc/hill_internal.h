@@ -24,7 +24,8 @@ struct ScoreArgs {
   int64_t q_sb, q_sh, k_sb, k_sh, k_sn;
   float* scores;      // RAW: per-token sums, may be NULL when accum is given
   float* accum;       // RAW: running importance (+=), may be NULL
-  float* logits;      // ATTN: [B][H][cap]
+  float* logits;      // ATTN: [B][H][lstride] (lstride = cap rounded up to 32: a warp's 32 tokens of a head fill one 128-byte line)
+  int64_t lstride;
   float2* partials;   // ATTN: [B][nslot][H] (max, sum 2^(z2 - max)), base-2 logits z2 = z * log2 e
   int nslot;          // = grid size of the launch x score_deal_warps(nkv, G) (one slot per warp share)
   int kvh;            // RAW with per-KV-head selection: scores/accum [B][Hkv][cap], summed over each group only
@@ -42,7 +43,8 @@ struct ScoreArgs {
 };
 
 struct FinalizeArgs {
-  const float* logits;
+  const float* logits;   // [B][H][lstride]; every line read is discarded from L2 afterwards (dead data)
+  int64_t lstride;
   const float2* partials;
   const int32_t* lens;
   int B, H, cap, nslot;
@@ -54,6 +56,7 @@ struct FinalizeArgs {
   int kvh;            // 1: scores/accum are [B][Hkv][cap], the sum over each KV head's G query heads
   int Hkv;
   float2* stats;      // [B][H] (max, 1/sum) per head, or NULL: every finalize CTA combines the partials
+  int tpt;            // blocks of 256 tokens per finalize CTA (set by the launcher)
 };
 
 struct QuantArgs {
@@ -72,6 +75,7 @@ struct SelectArgs {
   const int32_t* k;
   int B, cap, max_k;
   int chunk;          // filled by the launcher
+  int run;            // lean selection: keys per thread (filled by the launcher)
   const uint32_t* hist0;   // optional [B][2048]: counts of the leading 11-bit key digit (tokens j < len - recent)
   int rows_per_seq;   // key rows per sequence: 1, or Hkv with per-KV-head selection (row r reads lens/k of r / rows_per_seq)
   int recent;         // BKP: the most recent min(recent, len) tokens are kept outright (0: none)
@@ -156,8 +160,12 @@ int score_max_kv_heads();
 int score_deal_warps(int nkv, int G);
 cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8, bool deal, int grid,
                          cudaStream_t st);
-// Launches the normalisation (one or two kernels: *kernels is set to the count).
-cudaError_t launch_attn_finalize(const FinalizeArgs& a, int sms, cudaStream_t st, int* kernels);
+// Launches the normalisation (one or two kernels: *kernels is set to the
+// count).  two_kernel: always combine the partials in their own kernel first,
+// so that the finalize kernel takes its small form (at most 64 registers),
+// which fits beside a scoring CTA on one SM.
+cudaError_t launch_attn_finalize(const FinalizeArgs& a, int sms, cudaStream_t st, int* kernels,
+                                 bool two_kernel = false);
 
 // selftest.cu
 cudaError_t launch_selftest_wait(unsigned long long limit_ns, unsigned* err, cudaStream_t st);
@@ -170,6 +178,11 @@ int select_cluster_size(int cap);
 size_t select_smem_bytes(int cap, int C);
 int select_hist_bins();
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
+// The lean selection (same result as launch_select): a cluster of at most
+// 8 CTAs of 256 threads per key row, small enough to share an SM with the
+// scoring kernel; every key is read once from global memory.
+int select_lean_cluster_size(int cap);
+cudaError_t launch_select_lean(const SelectArgs& a, cudaStream_t st);
 
 // attn.cu
 int attn_batch_tokens();

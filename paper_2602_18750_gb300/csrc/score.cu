@@ -66,6 +66,11 @@ struct ScoreCfg {
 };
 
 constexpr int kL2Ahead = 4;   // stages per warp brought into L2 before the dependency wait
+// Registers per thread of the scoring kernel: at most 192, so that one CTA
+// of 256 threads at 64 registers (the two-kernel normalisation's finalize,
+// the lean selection) still fits beside it in the SM's 65536 registers and the
+// layer-pipelined evaluation can run them during the next layer's K stream.
+constexpr int kScoreMaxRegs = 192;
 
 __device__ __forceinline__ int find_seq(const int* tstart, int B, int item) {
   int lo = 0, hi = B;  // tstart[lo] <= item < tstart[hi]
@@ -88,7 +93,7 @@ struct Cursor {
 };
 
 template <int DT, int G, bool RAW, bool F8, bool DEAL>
-__global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_constant__ ScoreArgs a) {
+__global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_constant__ ScoreArgs a) {
   using Cfg = ScoreCfg<G, F8>;
   constexpr int kSlotBytes = Cfg::kSlotBytes;
   constexpr int kSW = Cfg::kSW;
@@ -161,6 +166,8 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
   const int it0 = (DEAL && ng == 0) ? it_hi : it_lo + sub;   // this warp's first item
 
   const uint64_t pol = l2_evict_first_policy();
+  // the logits stay in L2 until the normalisation reads (and discards) them
+  const uint64_t pol_keep = l2_evict_last_policy();
   const uint32_t stage0 = base_addr + warp * kSW * kSlotBytes;
   const uint32_t bar0 = base_addr + Cfg::kOffBar + warp * kSW * 8;
   const uint32_t scale0 = base_addr + Cfg::kOffScale + warp * kSW * kT * 4;   // F8 only
@@ -469,7 +476,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
           }
         }
       } else {
-        float* lg = a.logits + ((int64_t)b * H + g * a.Gs + a.hoff) * cap + j0;
+        float* lg = a.logits + ((int64_t)b * H + g * a.Gs + a.hoff) * a.lstride + j0;
 #pragma unroll
         for (int c = 0; c < kCols; ++c) {
           const int hl = 2 * tig + c;
@@ -479,7 +486,7 @@ __global__ void __launch_bounds__(kThreads, 1) hill_score_kernel(const __grid_co
             const int mb = u >> 1, e = (u & 1) * 2 + c;
             const int t = mb * 16 + grp + (u & 1) * 8;
             z[u] = t < nv ? acc[mb][e] * kLog2eInvSqrtD : -INFINITY;
-            if (t < nv && hl < Gn) lg[(int64_t)hl * cap + t] = z[u];
+            if (t < nv && hl < Gn) st_global_hint(lg + (int64_t)hl * a.lstride + t, z[u], pol_keep);
           }
           const float mn = fmaxf(st_m[r][c], fmaxf(fmaxf(z[0], z[1]), fmaxf(z[2], z[3])));
           st_l[r][c] = st_l[r][c] * ex2(st_m[r][c] - mn) +
@@ -536,6 +543,7 @@ constexpr int kFinPartMax = 32;                    // partials per thread held i
 constexpr int kFinPartFew = 4;                     // the same when a sequence has few (<= 32) slots
 constexpr int kHistBins = 2048;                    // leading 11 bits of the order-preserving key
 constexpr int kFinZReg = 32;                       // logits per token held in registers
+constexpr int kFinMaxTpt = 16;                     // token blocks per CTA at most (split step)
 
 // Combine the ns per-CTA partials (max, sum) of every head of sequence b into
 // mh[h] (max) and il[h] (1 / sum): kFinPartThreads threads per head, each
@@ -600,7 +608,8 @@ __global__ void __launch_bounds__(kFinThreads, STATS ? 4 : 2) hill_attn_finalize
   const int b = blockIdx.y;
   int len = a.lens[b];
   len = len < 0 ? 0 : (len > a.cap ? a.cap : len);
-  const int jb = blockIdx.x * kFinChunk;
+  // this CTA's tokens: a.tpt blocks of kFinChunk from jb
+  const int jb = blockIdx.x * kFinChunk * a.tpt;
   if (jb >= len) return;
   // the scoring CTAs that met b wrote slots 0 .. ns-1
   // (every thread counts the tiles of a share of the sequences)
@@ -629,12 +638,12 @@ __global__ void __launch_bounds__(kFinThreads, STATS ? 4 : 2) hill_attn_finalize
   pdl_launch_dependents();
   // this token's logits of the first kFinZReg heads, loaded before the
   // partials are combined so that both round trips overlap
-  const int j = jb + threadIdx.x;
-  const bool valid = j < len;
-  const float* zp = a.logits + (int64_t)b * a.H * a.cap + j;
+  int j = jb + threadIdx.x;
+  bool valid = j < len;
+  const float* zp = a.logits + (int64_t)b * a.H * a.lstride + j;
   float zr[kFinZReg];
 #pragma unroll
-  for (int u = 0; u < kFinZReg; ++u) zr[u] = (valid && u < a.H) ? zp[(int64_t)u * a.cap] : 0.f;
+  for (int u = 0; u < kFinZReg; ++u) zr[u] = (valid && u < a.H) ? zp[(int64_t)u * a.lstride] : 0.f;
   if constexpr (STATS) {
     for (int h = threadIdx.x; h < a.H; h += kFinThreads) {
       const float2 st = a.stats[(int64_t)b * a.H + h];
@@ -650,6 +659,7 @@ __global__ void __launch_bounds__(kFinThreads, STATS ? 4 : 2) hill_attn_finalize
   if (a.hist0)
     for (int i = threadIdx.x; i < kHistBins; i += kFinThreads) hcount[i] = 0u;
   __syncthreads();
+  for (int blk = 0;;) {   // the CTA's token blocks (one unless a.tpt > 1)
   if (KVH && valid) {
     // per-KV-head importance: the sum over each group of G query heads,
     // stored as soon as the group is complete (heads of a group are adjacent)
@@ -675,7 +685,7 @@ __global__ void __launch_bounds__(kFinThreads, STATS ? 4 : 2) hill_attn_finalize
     for (int h = kFinZReg; h < a.H; h += 16) {
       float z[16];
 #pragma unroll
-      for (int u = 0; u < 16; ++u) z[u] = h + u < a.H ? zp[(int64_t)(h + u) * a.cap] : 0.f;
+      for (int u = 0; u < 16; ++u) z[u] = h + u < a.H ? zp[(int64_t)(h + u) * a.lstride] : 0.f;
 #pragma unroll
       for (int u = 0; u < 16; ++u)
         if (h + u < a.H) {
@@ -697,11 +707,11 @@ __global__ void __launch_bounds__(kFinThreads, STATS ? 4 : 2) hill_attn_finalize
     for (; h + 16 <= a.H; h += 16) {
       float z[16];
 #pragma unroll
-      for (int u = 0; u < 16; ++u) z[u] = zp[(int64_t)(h + u) * a.cap];
+      for (int u = 0; u < 16; ++u) z[u] = zp[(int64_t)(h + u) * a.lstride];
 #pragma unroll
       for (int u = 0; u < 16; ++u) s += ex2(z[u] - mh[h + u]) * il[h + u];
     }
-    for (; h < a.H; ++h) s += ex2(zp[(int64_t)h * a.cap] - mh[h]) * il[h];
+    for (; h < a.H; ++h) s += ex2(zp[(int64_t)h * a.lstride] - mh[h]) * il[h];
     const int64_t o = (int64_t)b * a.cap + j;
     if (a.scores) a.scores[o] = s;
     float key = s;
@@ -710,6 +720,24 @@ __global__ void __launch_bounds__(kFinThreads, STATS ? 4 : 2) hill_attn_finalize
       a.accum[o] = key;
     }
     if (a.hist0 && j < len - min(a.recent, len)) atomicAdd(&hcount[ordered_key(key) >> 21], 1u);
+  }
+  // The logits are dead once read: drop this warp's lines from L2 without
+  // writing them back (each 128-byte line holds the warp's 32 tokens of one
+  // head; every lane has consumed its loads before the warp passes the sync).
+  {
+    const int j0 = j - (int)(threadIdx.x & 31);
+    __syncwarp();
+    if (j0 < len)
+      for (int h = threadIdx.x & 31; h < a.H; h += 32)
+        l2_discard_line(a.logits + ((int64_t)b * a.H + h) * a.lstride + j0);
+  }
+  // the next block of tokens (its logits loaded before they are used)
+  if (++blk >= a.tpt || jb + blk * kFinChunk >= len) break;
+  j = jb + blk * kFinChunk + threadIdx.x;
+  valid = j < len;
+  zp = a.logits + (int64_t)b * a.H * a.lstride + j;
+#pragma unroll
+  for (int u = 0; u < kFinZReg; ++u) zr[u] = (valid && u < a.H) ? zp[(int64_t)u * a.lstride] : 0.f;
   }
   if (a.hist0) {
     __syncthreads();
@@ -836,12 +864,23 @@ cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8
   return f8 ? launch_score_m<1, true>(a, G, raw, deal, grid, st) : launch_score_m<1, false>(a, G, raw, deal, grid, st);
 }
 
-cudaError_t launch_attn_finalize(const FinalizeArgs& a, int sms, cudaStream_t st, int* kernels) {
-  dim3 grid((a.cap + kFinChunk - 1) / kFinChunk, a.B);
+cudaError_t launch_attn_finalize(const FinalizeArgs& a0, int sms, cudaStream_t st, int* kernels,
+                                 bool two_kernel) {
+  FinalizeArgs a = a0;
+  a.tpt = 1;
+  // The split step's normalisation runs beside the next layer's scoring
+  // kernel, which leaves room for about one such CTA per SM: each thread
+  // takes several tokens so that the grid needs at most about two rounds of
+  // CTAs instead of trickling through in many.
+  if (two_kernel)
+    while (a.tpt < kFinMaxTpt &&
+           (long long)a.B * ((a.cap + kFinChunk * a.tpt - 1) / (kFinChunk * a.tpt)) > 2LL * sms)
+      a.tpt <<= 1;
+  dim3 grid((a.cap + kFinChunk * a.tpt - 1) / (kFinChunk * a.tpt), a.B);
   const size_t smem = 2 * a.H * sizeof(float) + (a.hist0 ? kHistBins * sizeof(uint32_t) : 0);
   // more than two normalisation CTAs per SM: combine the partials once per
   // (b, h) in a kernel of their own instead of once per CTA
-  if (a.stats && (long long)grid.x * grid.y > 2LL * sms) {
+  if (a.stats && (two_kernel || (long long)grid.x * grid.y > 2LL * sms)) {
     *kernels = 2;
     const int pairs = a.B * a.H;
     cudaError_t e = launch_pdl(hill_attn_stats_kernel, dim3((pairs + kStatsWarps - 1) / kStatsWarps),

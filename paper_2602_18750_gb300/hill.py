@@ -9,7 +9,7 @@ fails loudly if the library has not been built.
 Names follow the C ABI: :func:`hill_score`, :func:`hill_topk_select`,
 :func:`hill_gather_sparse_attn`, :func:`hill_evict_step`, :func:`hill_topk_select_bkp`,
 :func:`hill_evict_step_bkp`, :func:`hill_quantize_k`, :func:`hill_score_f8`, :func:`hill_evict_step_f8`,
-:func:`hill_evict_step_kvh`,
+:func:`hill_evict_step_kvh`, :func:`hill_evict_step_begin`, :func:`hill_evict_step_end`,
 :func:`hill_workspace_bytes`, :func:`hill_sync_status`.
 """
 from __future__ import annotations
@@ -76,6 +76,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_evict_step_bkp.argtypes = [D, P, P, P, P, P, I32, I32, I32, P, P, P, P, P, P, P, SZ, P]
     lib.hill_quantize_k.argtypes = [D, P, P, P, I32, P, P, P]
     lib.hill_evict_step_kvh.argtypes = [D, P, P, P, P, P, I32, I32, P, P, P, P, P, P, SZ, P]
+    lib.hill_evict_step_begin.argtypes = [D, P, P, P, I32, I32, P, P, P, SZ, P]
+    lib.hill_evict_step_end.argtypes = [D, P, P, I32, I32, I32, P, P, P, P, P, P, SZ, P]
     lib.hill_selftest_wait.argtypes = [ctypes.c_uint32, P]
     lib.hill_score_f8.argtypes = [D, P, P, P, P, I32, P, P, P, SZ, P]
     lib.hill_evict_step_f8.argtypes = [D, P, P, P, P, P, P, P, I32, I32, P, P, P, P, P, P, SZ, P]
@@ -88,7 +90,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_kernel_launches.restype = ctypes.c_uint64
     for name in ("hill_score", "hill_topk_select", "hill_gather_sparse_attn", "hill_evict_step",
                  "hill_topk_select_bkp", "hill_evict_step_bkp", "hill_quantize_k", "hill_score_f8",
-                 "hill_evict_step_f8", "hill_evict_step_kvh", "hill_selftest_wait", "hill_sync_status"):
+                 "hill_evict_step_f8", "hill_evict_step_kvh", "hill_evict_step_begin", "hill_evict_step_end",
+                 "hill_selftest_wait", "hill_sync_status"):
         getattr(lib, name).restype = I32
     _lib = lib
     return lib
@@ -209,6 +212,23 @@ def hill_evict_step_bkp(desc, q, k_cache, v_cache, lens, k, recent, max_k, mode,
                                       _ptr(k), int(recent), int(max_k), int(mode), _ptr(accum), _ptr(scores),
                                       _ptr(idx), _ptr(count), _ptr(hits), _ptr(out), wp, wn,
                                       _stream(stream)), "hill_evict_step_bkp")
+
+
+def hill_evict_step_begin(desc, q, k_cache, lens, max_k, mode, accum, scores, ws, stream=None) -> None:
+    """First half of the split step: the scoring kernel (K stream)."""
+    wp, wn = _ws(ws)
+    _check(load().hill_evict_step_begin(ctypes.byref(desc), _ptr(q), _ptr(k_cache), _ptr(lens), int(max_k),
+                                        int(mode), _ptr(accum), _ptr(scores), wp, wn, _stream(stream)),
+           "hill_evict_step_begin")
+
+
+def hill_evict_step_end(desc, lens, k, max_k, mode, accum, scores, idx, count, ws, recent=0, hits=None,
+                        stream=None) -> None:
+    """Second half of the split step: normalisation (ATTN) and selection."""
+    wp, wn = _ws(ws)
+    _check(load().hill_evict_step_end(ctypes.byref(desc), _ptr(lens), _ptr(k), int(recent), int(max_k), int(mode),
+                                      _ptr(accum), _ptr(scores), _ptr(idx), _ptr(count), _ptr(hits), wp, wn,
+                                      _stream(stream)), "hill_evict_step_end")
 
 
 def hill_evict_step_kvh(desc, q, k_cache, v_cache, lens, k, max_k, mode, accum, scores, idx, count, out, ws,
