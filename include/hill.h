@@ -182,10 +182,9 @@ hill_status hill_evict_step_bkp(const hill_desc* desc, const void* q, const void
  * normalisation (scores, accum += as in hill_score), then the top-k selection
  * of hill_topk_select_bkp (recent = 0 and hits = NULL: exactly
  * hill_topk_select) on accum if given, else on this step's scores.  It reads
- * no keys.  Its kernels are sized to share the GPU's multiprocessors with a
- * scoring kernel running at the same time (the selection runs as clusters of
- * at most 8 CTAs of 256 threads per sequence, re-reading the keys from
- * global memory).
+ * no keys.  Its kernels run beside a scoring kernel of another layer: the
+ * normalisation's finalize fits next to a scoring CTA on one SM, and the
+ * selection uses the SMs the scoring grid of begin leaves free.
  *
  * Both calls of one step take the same desc, lens, max_k, mode, accum,
  * scores and ws (sized by hill_workspace_bytes); end may be issued on another
@@ -195,10 +194,11 @@ hill_status hill_evict_step_bkp(const hill_desc* desc, const void* q, const void
  * end of layer l (three let the K stream run two layers ahead of the
  * selection).  The scoring kernel of begin takes four fifths of the SMs, so
  * that end's kernels have room beside it.  Results equal those of
- * hill_evict_step_bkp without attention (scores within rounding: the split
- * normalisation always combines the softmax partials in a kernel of its own;
- * selections follow the same rule).  Attention: hill_gather_sparse_attn on idx
- * and count afterwards. */
+ * hill_evict_step_bkp without attention, the ATTN scores within rounding (the
+ * smaller scoring grid and the two-kernel normalisation combine the softmax
+ * partials in another order); the selection follows the same rule on the
+ * step's own scores.  Attention: hill_gather_sparse_attn on idx and count
+ * afterwards. */
 hill_status hill_evict_step_begin(const hill_desc* desc, const void* q, const void* k_cache,
                                   const int32_t* lens, int32_t max_k, hill_score_mode mode, float* accum,
                                   float* scores, void* ws, size_t ws_bytes, void* stream);

@@ -346,7 +346,7 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
 hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens, const int32_t* k,
                        int max_k, int32_t* idx, int32_t* count, const DeviceInfo& di, cudaStream_t st,
                        const uint32_t* hist0 = nullptr, int recent = 0, uint16_t* hits = nullptr,
-                       bool kvh = false, bool lean = false) {
+                       bool kvh = false) {
   if (d->batch == 0) return HILL_OK;
   SelectArgs a{};
   a.key = key;
@@ -362,7 +362,7 @@ hill_status run_select(const hill_desc* d, const float* key, const int32_t* lens
   a.hits = hits;
   a.rows_per_seq = kvh ? d->num_kv_heads : 1;
   a.err = di.err;
-  return from_cuda(counted(lean ? launch_select_lean(a, st) : launch_select(a, st), 1));
+  return from_cuda(counted(launch_select(a, st), 1));
 }
 
 hill_status run_attn(const hill_desc* d, const void* q, const void* k, const void* v, const int32_t* idx,
@@ -588,8 +588,7 @@ hill_status hill_evict_step_end(const hill_desc* desc, const int32_t* lens, cons
                   kScoreNormalise);
     if (s != HILL_OK) return s;
   }
-  return run_select(desc, accum ? accum : s_out, lens, k, max_k, idx, count, di, st, hist0, recent, hits, false,
-                    true);
+  return run_select(desc, accum ? accum : s_out, lens, k, max_k, idx, count, di, st, hist0, recent, hits);
 }
 
 hill_status hill_evict_step_kvh(const hill_desc* desc, const void* q, const void* k_cache, const void* v_cache,

@@ -75,7 +75,6 @@ struct SelectArgs {
   const int32_t* k;
   int B, cap, max_k;
   int chunk;          // filled by the launcher
-  int run;            // lean selection: keys per thread (filled by the launcher)
   const uint32_t* hist0;   // optional [B][2048]: counts of the leading 11-bit key digit (tokens j < len - recent)
   int rows_per_seq;   // key rows per sequence: 1, or Hkv with per-KV-head selection (row r reads lens/k of r / rows_per_seq)
   int recent;         // BKP: the most recent min(recent, len) tokens are kept outright (0: none)
@@ -178,11 +177,7 @@ int select_cluster_size(int cap);
 size_t select_smem_bytes(int cap, int C);
 int select_hist_bins();
 cudaError_t launch_select(const SelectArgs& a, cudaStream_t st);
-// The lean selection (same result as launch_select): a cluster of at most
-// 8 CTAs of 256 threads per key row, small enough to share an SM with the
-// scoring kernel; every key is read once from global memory.
-int select_lean_cluster_size(int cap);
-cudaError_t launch_select_lean(const SelectArgs& a, cudaStream_t st);
+
 
 // attn.cu
 int attn_batch_tokens();

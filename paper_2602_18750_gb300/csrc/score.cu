@@ -67,9 +67,9 @@ struct ScoreCfg {
 
 constexpr int kL2Ahead = 4;   // stages per warp brought into L2 before the dependency wait
 // Registers per thread of the scoring kernel: at most 192, so that one CTA
-// of 256 threads at 64 registers (the two-kernel normalisation's finalize,
-// the lean selection) still fits beside it in the SM's 65536 registers and the
-// layer-pipelined evaluation can run them during the next layer's K stream.
+// of 256 threads at 64 registers (the two-kernel normalisation's finalize)
+// still fits beside it in the SM's 65536 registers and the layer-pipelined
+// evaluation can run it during the next layer's K stream.
 constexpr int kScoreMaxRegs = 192;
 
 __device__ __forceinline__ int find_seq(const int* tstart, int B, int item) {

@@ -1,12 +1,11 @@
 """GPU parity of the split step (hill_evict_step_begin / hill_evict_step_end),
-the building block of the layer-pipelined evaluation (Sec. 4.3), and of the
-lean selection kernel it runs:
+the building block of the layer-pipelined evaluation (Sec. 4.3):
 
-* the lean selection alone (RAW mode: end() selects on the caller's scores)
-  against the oracle's sort of the same keys, bit for bit: cluster sizes 1
-  to 8, heavy exact ties, signed zeros, flat key distributions whose crossing
-  bucket is too large to gather (the cluster-histogram path), BKP windows and
-  hit tables, and the budget edge cases;
+* the selection of end() alone (RAW mode: end() selects on the caller's
+  scores, building the leading-digit histogram itself) against the oracle's
+  sort of the same keys, bit for bit: cluster sizes 1 to 8, heavy exact ties,
+  signed zeros, flat key distributions with large crossing buckets, BKP
+  windows and hit tables, and the budget edge cases;
 * the split step against the oracle (scores, selection by the gap rule) and
   against the fused hill_evict_step (RAW: bit for bit; ATTN: scores within
   the tolerance, since the split step's scoring grid -- four fifths of the
@@ -42,8 +41,8 @@ def _i32(x):
     return torch.tensor(x, dtype=torch.int32, device="cuda")
 
 
-def _lean_select(H, s, lens, k, max_k, recent=0, hits=None):
-    """end() in RAW mode: the lean selection on the caller's keys s [B][cap]."""
+def _end_select(H, s, lens, k, max_k, recent=0, hits=None):
+    """end() in RAW mode: the selection on the caller's keys s [B][cap]."""
     B, cap = s.shape
     q = torch.zeros(B, 4, 128, dtype=torch.float16, device="cuda")
     K = torch.zeros(B, 4, 8, 128, dtype=torch.float16, device="cuda")
@@ -74,33 +73,33 @@ def _keys(kind, B, cap, seed):
 
 @pytest.mark.parametrize("kind", ["lognormal", "uniform", "ties", "softmaxlike"])
 @pytest.mark.parametrize("cap", [700, 4096, 5000, 12000, 40000, 131079])
-def test_lean_select_matches_oracle(H, oracle_mod, kind, cap):
-    """Clusters of 1, 2, 4 and 8 CTAs (4096 keys per CTA at most before the
-    cluster doubles); budgets from one token to most of the sequence."""
+def test_end_select_matches_oracle(H, oracle_mod, kind, cap):
+    """One CTA and clusters of 2, 4 and 8 CTAs per row; budgets from one
+    token to most of the sequence."""
     B = 3
     s = _keys(kind, B, cap, cap + len(kind))
     lens = [cap, cap - 37, max(1, cap // 3)]
     k = [max(1, cap // 10), 1, lens[2] - 1]
     max_k = max(k) + 3
-    idx, cnt = _lean_select(H, s, lens, k, max_k)
+    idx, cnt = _end_select(H, s, lens, k, max_k)
     H.hill_sync_status()
     idx_o, cnt_o, _ = oracle_mod.topk(s.numpy().astype(np.float64), lens, k, max_k)
     assert np.array_equal(cnt.cpu().numpy(), cnt_o)
     assert np.array_equal(idx.cpu().numpy(), idx_o)
 
 
-def test_lean_select_budget_edges(H, oracle_mod):
+def test_end_select_budget_edges(H, oracle_mod):
     """k = 0, k = len, k > len, empty and one-token sequences, and a budget
     above max_k (count capped, device error word raised)."""
     cap = 9000
     s = _keys("lognormal", 5, cap, 3)
     lens = [cap, 0, 1, 5000, 8000]
     k = [0, 4, 1, 5000, 9999]
-    idx, cnt = _lean_select(H, s, lens, k, 9000)
+    idx, cnt = _end_select(H, s, lens, k, 9000)
     H.hill_sync_status()
     idx_o, cnt_o, _ = oracle_mod.topk(s.numpy().astype(np.float64), lens, k, 9000)
     assert np.array_equal(cnt.cpu().numpy(), cnt_o) and np.array_equal(idx.cpu().numpy(), idx_o)
-    idx, cnt = _lean_select(H, s, [cap] * 5, [100, 20, 30, 40, 50], 32)
+    idx, cnt = _end_select(H, s, [cap] * 5, [100, 20, 30, 40, 50], 32)
     with pytest.raises(H.HillError) as ei:
         H.hill_sync_status()
     assert ei.value.status == H.HILL_ERR_DEVICE
@@ -110,8 +109,8 @@ def test_lean_select_budget_edges(H, oracle_mod):
 
 @pytest.mark.parametrize("recent", [0, 37, 4000])
 @pytest.mark.parametrize("cap", [3000, 40000])
-def test_lean_select_bkp_window_and_hits(H, oracle_mod, recent, cap):
-    """The pinned window and the hit-rate table (Sec. 4.2) of the lean
+def test_end_select_bkp_window_and_hits(H, oracle_mod, recent, cap):
+    """The pinned window and the hit-rate table (Sec. 4.2) of end()'s
     selection equal the oracle's BKP selection over three steps."""
     B = 2
     lens = [cap, cap // 2 + 11]
@@ -121,7 +120,7 @@ def test_lean_select_bkp_window_and_hits(H, oracle_mod, recent, cap):
     hits_ref = np.zeros((B, cap), dtype=np.uint16)
     for step in range(3):
         s = _keys("lognormal", B, cap, 100 * step + cap)
-        idx, cnt = _lean_select(H, s, lens, k, max_k, recent=recent, hits=hits)
+        idx, cnt = _end_select(H, s, lens, k, max_k, recent=recent, hits=hits)
         H.hill_sync_status()
         idx_o, cnt_o, _, hits_ref = oracle_mod.bkp_select(s.numpy().astype(np.float64), lens, k, recent, max_k,
                                                           hits_ref)
@@ -161,7 +160,7 @@ def test_split_step_matches_oracle_and_fused(H, oracle_mod, mode, shape):
     ref = oracle_mod.evict_step(mode, q.cpu(), K.cpu(), V.cpu(), lens, k, max_k, with_attn=False)
     check_scores(scores.cpu().numpy(), ref["s"], lens)
     check_selection(idx.cpu().numpy(), cnt.cpu().numpy(), ref["s"], lens, k, max_k)
-    # the lean selection is exact on its own keys
+    # the selection is exact on its own keys
     idx_o, cnt_o, _ = oracle_mod.topk(scores.cpu().numpy().astype(np.float64), lens, k, max_k)
     assert np.array_equal(idx.cpu().numpy(), idx_o) and np.array_equal(cnt.cpu().numpy(), cnt_o)
     # the fused step: RAW sums do not depend on the grid (bit-identical
