@@ -608,17 +608,20 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-def eval_select_only(args, n, hill, dev, world, mode):
-    """Evaluation + selection alone (no attention) on workload n with all its
-    layers resident (as many as fit), in the layer-pipelined form and
-    serially, one CUDA graph per decode step over all layers, timed like the
-    main region; plus the scoring stage (hill_score) per launch.  Used for the
-    contexts of 32K tokens or more that the headline workload does not cover."""
-    rank, _, local = dist_env()
-    w, _ = workload_for(n, replica_seed(args.seed, rank), None)
+def measure_workload(args, w, hill, dev, world, mode, full_step=False, layers_resident=None):
+    """Evaluation + selection alone (no attention) on workload w with as many
+    layers resident as fit (or `layers_resident`), in the layer-pipelined form
+    and serially, one CUDA graph per decode step over all layers, timed like
+    the main region; the scoring stage (hill_score) per launch; and with
+    full_step the pipelined step with the sparse attention.  Accumulating
+    workloads carry their running importance across the timed steps."""
+    _, _, local = dist_env()
     L, S, B, Hq, Hkv, d = w.layers, w.steps, w.batch, w.heads, w.kv_heads, w.head_dim
     per_layer = 2 * B * Hkv * w.capacity * d * torch.finfo(w.dtype).bits // 8
     lres = max(1, min(L, int(0.7 * torch.cuda.mem_get_info(dev)[0]) // per_layer))
+    if layers_resident:
+        lres = min(lres, layers_resident)
+    t_gen = time.time()
     Kall = torch.empty(lres, B, Hkv, w.capacity, d, dtype=w.dtype, device=dev)
     Vall = torch.empty_like(Kall)
     for l in range(lres):
@@ -626,55 +629,73 @@ def eval_select_only(args, n, hill, dev, world, mode):
         Kall[l].copy_(K)
         Vall[l].copy_(V)
         del K, V
-    q_all = torch.stack([torch.stack([inputs.step_query(w, l, t, device=dev) for l in range(L)]) for t in range(S)])
-    lens_all = torch.tensor([w.lens_at(t) for t in range(S)], dtype=torch.int32, device=dev)
-    k_all = torch.tensor([w.budget_at(t) for t in range(S)], dtype=torch.int32, device=dev)
+    order = [(args.warmup + i) % S for i in range(args.steps)]
+    steps_used = sorted(set(order) | set(i % S for i in range(args.warmup)))
+    q_all = {t: torch.stack([inputs.step_query(w, l, t, device=dev) for l in range(L)]) for t in steps_used}
+    lens_all = {t: torch.tensor(w.lens_at(t), dtype=torch.int32, device=dev) for t in steps_used}
+    k_all = {t: torch.tensor(w.budget_at(t), dtype=torch.int32, device=dev) for t in steps_used}
     accum = torch.zeros(lres, B, w.capacity, dtype=torch.float32, device=dev) if w.accumulate else None
     scores = torch.empty(L, B, w.capacity, dtype=torch.float32, device=dev)
     idx = torch.empty(L, B, w.max_k, dtype=torch.int32, device=dev)
     count = torch.empty(L, B, dtype=torch.int32, device=dev)
-    desc = hill.make_desc(q_all[0, 0], Kall[0], Vall[0])
+    out = torch.empty(L, B, Hq, d, dtype=torch.float32, device=dev) if full_step else None
+    desc = hill.make_desc(q_all[steps_used[0]][0], Kall[0], Vall[0])
     wss = [hill.alloc_workspace(desc, mode, w.max_k, dev) for _ in range(SPLIT_WORKSPACES)]
-    stream, side = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    wsa = [hill.alloc_workspace(desc, mode, w.max_k, dev) for _ in range(2)] if full_step else None
+    stream, side, att = (torch.cuda.Stream(device=dev) for _ in range(3))
     torch.cuda.synchronize(dev)   # the inputs were made on the default stream
+    t_gen = time.time() - t_gen
 
     def acc(l):
         return accum[l % lres] if accum is not None else None
 
-    def issue(t, st, frm):
-        def fused(l, _, s_, wi):
-            hill.hill_evict_step(desc, q_all[t, l], Kall[l % lres], Vall[l % lres], lens_all[t], k_all[t], w.max_k,
-                                 mode, acc(l), scores[l], idx[l], count[l], None, wss[wi], s_)
+    def issue(t, st, frm, with_attn):
+        def fused(l, a_, s_, wi):
+            hill.hill_evict_step(desc, q_all[t][l], Kall[l % lres], Vall[l % lres], lens_all[t], k_all[t], w.max_k,
+                                 mode, acc(l), scores[l], idx[l], count[l], out[l] if a_ else None, wss[wi], s_)
 
         def begin(l, s_, wi):
-            hill.hill_evict_step_begin(desc, q_all[t, l], Kall[l % lres], lens_all[t], w.max_k, mode, acc(l),
+            hill.hill_evict_step_begin(desc, q_all[t][l], Kall[l % lres], lens_all[t], w.max_k, mode, acc(l),
                                        scores[l], wss[wi], s_)
 
         def end(l, s_, wi):
             hill.hill_evict_step_end(desc, lens_all[t], k_all[t], w.max_k, mode, acc(l), scores[l], idx[l],
                                      count[l], wss[wi], stream=s_)
 
-        issue_layers(frm, L, st, side, None, False, fused, begin, end, None)
+        def attn(l, s_, wi):
+            hill.hill_gather_sparse_attn(desc, q_all[t][l], Kall[l % lres], Vall[l % lres], idx[l], count[l],
+                                         w.max_k, out[l], wsa[wi], s_)
 
-    order = [(args.warmup + i) % S for i in range(args.steps)]
+        issue_layers(frm, L, st, side, att, with_attn, fused, begin, end, attn)
+
     tokens = sum(L * sum(w.lens_at(t)) for t in order)
     peak, _ = measured_peaks()
     piped = pipelined_form(False, mode, w.accumulate, lres)
-    forms = {}
-    for frm in dict.fromkeys([piped, "serial"]):
+    runs = [(piped, False), ("serial", False)] + ([(piped, True)] if full_step else [])
+    res = {}
+    for frm, with_attn in dict.fromkeys(runs):
         with torch.cuda.stream(stream):
-            issue(0, stream, frm)
+            issue(steps_used[0], stream, frm, with_attn)
         hill.hill_sync_status(stream)
-        graphs = capture_steps(S, stream, lambda t, st: issue(t, st, frm))
+        graphs = [None] * S
+        for t in steps_used:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                issue(t, stream, frm, with_attn)
+            graphs[t] = g
         if accum is not None:
             accum.zero_()
         ms, clock_info = time_replays(graphs, order, args.warmup, stream, dev, clocks_of=local)
         ms = max_over_ranks(ms, dev)
         hill.hill_sync_status(stream)
         del graphs
-        forms[frm] = dict(eval_summary(ms, tokens, Hkv * d * 2, len(order) * L, world, peak, frm), clocks=clock_info)
-    # the scoring stage alone, per launch, at the last decode step
-    t_s = S - 1
+        if with_attn:
+            res["step"] = {"schedule": SCHEDULES[frm], "us_per_layer": round(ms * 1e3 / (len(order) * L), 2),
+                           "tokens_per_s": round(world * tokens / (ms / 1e3), 1), "clocks": clock_info}
+        else:
+            res[frm] = dict(eval_summary(ms, tokens, Hkv * d * 2, len(order) * L, world, peak, frm), clocks=clock_info)
+    # the scoring stage alone, per launch, at the last timed decode step
+    t_s = order[-1]
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(L)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(L)]
     with torch.cuda.stream(stream):
@@ -682,26 +703,71 @@ def eval_select_only(args, n, hill, dev, world, mode):
             for l in range(L):
                 if rep == 1:
                     starts[l].record(stream)
-                hill.hill_score(desc, q_all[t_s, l], Kall[l % lres], lens_all[t_s], mode, scores[l], None, wss[0],
+                hill.hill_score(desc, q_all[t_s][l], Kall[l % lres], lens_all[t_s], mode, scores[l], None, wss[0],
                                 stream)
                 if rep == 1:
                     ends[l].record(stream)
     stream.synchronize()
     hill.hill_sync_status(stream)
     score_us = sum(a.elapsed_time(b) for a, b in zip(starts, ends)) / L * 1e3
-    out = dict(forms[piped])
+    out_d = dict(res[piped])
     if piped != "serial":
-        out["serial"] = forms["serial"]
-    out.update({
+        out_d["serial"] = res["serial"]
+    if full_step:
+        out_d["step"] = res["step"]
+    out_d.update({
         "workload": w.name, "batch": B, "heads": Hq, "kv_heads": Hkv, "kv_dtype": str(w.dtype).replace("torch.", ""),
-        "tokens_last_step": w.lens_at(S - 1), "layers_resident": lres, "steps_timed": len(order),
+        "tokens_last_step": w.lens_at(S - 1), "budget": f"floor({w.budget_frac}*len)" if w.budget_tokens is None
+        else w.budget_tokens, "accumulate": w.accumulate, "layers": L, "layers_resident": lres,
+        "decode_steps": S, "steps_timed": len(order),
         "scoring_stage_us": round(score_us, 2),
         "scoring_stage_frac_of_measured_hbm": round(
             sum(w.lens_at(t_s)) * (Hkv * d * 2 + 4) / (score_us / 1e6) / 1e9 / peak, 4),
+        "generate_s": round(t_gen, 1),
     })
-    del Kall, Vall, q_all, accum, scores, idx, count, wss
+    del Kall, Vall, q_all, accum, scores, idx, count, out, wss, wsa
     torch.cuda.empty_cache()
-    return out
+    return out_d
+
+
+def eval_select_only(args, n, hill, dev, world, mode):
+    """The acceptance measurement of workload n (the contexts of 32K tokens
+    or more the headline workload does not cover)."""
+    rank, _, _ = dist_env()
+    w, _ = workload_for(n, replica_seed(args.seed, rank), None)
+    return measure_workload(args, w, hill, dev, world, mode)
+
+
+def run_sweep(args):
+    """The budget/batch sweep: B in {1, 8, 16} x {8K, 64K} tokens x budget in
+    {5, 10, 20, 50} %, 32 layers, cumulative importance across decode steps;
+    one JSON line per point (rank 0), resident layers reused cyclically where
+    the point's KV does not fit in HBM."""
+    import torch.distributed as dist
+
+    from paper_2602_18750_gb300 import build as hbuild
+    from paper_2602_18750_gb300 import hill
+
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    hbuild.build()
+    hill.load()
+    mode = hill.HILL_SCORE_ATTN if args.mode == "attn" else hill.HILL_SCORE_RAW
+    for B in inputs.SWEEP_BATCHES:
+        for n in inputs.SWEEP_LENS:
+            for frac in inputs.SWEEP_BUDGETS:
+                w = inputs.sweep_point(B, n, frac, seed=replica_seed(args.seed, rank))
+                r = measure_workload(args, w, hill, dev, world, mode, full_step=True,
+                                     layers_resident=args.layers_resident)
+                if rank == 0:
+                    print(json.dumps({"sweep_point": {"batch": B, "tokens": n, "budget_frac": frac},
+                                      "metric": METRIC, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                                      "warmup": args.warmup, "importance": args.mode, **r}), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
 
 
 def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all, accum, scores, idx, count,
@@ -960,6 +1026,8 @@ def main(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="the budget/batch sweep (B x tokens x budget, accumulating): one JSON line per point")
     ap.add_argument("--no-acceptance", action="store_true",
                     help="skip timing evaluation + selection on the other 32K+ workloads")
     ap.add_argument("--serial", action="store_true",
@@ -975,6 +1043,8 @@ def main(argv=None):
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":
         run_reference(args)
+    elif args.sweep:
+        run_sweep(args)
     else:
         run_ours(args)
 
