@@ -26,6 +26,7 @@ cores on the same workload and metric.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import math
@@ -324,8 +325,13 @@ def profile_traffic(kernel_key: str, workload: str):
     return None
 
 
-def workload_for(n: int, seed: int, layers_resident: int | None):
+def workload_for(n: int, seed: int, layers_resident: int | None, kv_heads: int | None = None):
     w = inputs.config(n, seed=seed)
+    if kv_heads:
+        # another head layout of the same workload: its query heads over kv_heads KV heads
+        if w.heads % kv_heads:
+            raise SystemExit(f"--kv-heads {kv_heads} does not divide {w.heads} query heads")
+        w = dataclasses.replace(w, kv_heads=kv_heads, name=f"{w.name}-kv{kv_heads}")
     lres = w.layers
     if layers_resident:
         lres = min(lres, layers_resident)
@@ -362,7 +368,7 @@ def run_ours(args):
     hill.load()
 
     mode = hill.HILL_SCORE_ATTN if args.mode == "attn" else hill.HILL_SCORE_RAW
-    w, lres = workload_for(args.workload, replica_seed(args.seed, rank), args.layers_resident)
+    w, lres = workload_for(args.workload, replica_seed(args.seed, rank), args.layers_resident, args.kv_heads)
     if args.layers_resident is None:
         # keep as many layers resident as fit in 70 % of the free device memory
         # (the 64K sweep point needs 8.6 GB of K/V per layer); layers beyond
@@ -976,7 +982,7 @@ def run_reference(args):
     if rank != 0:
         return
     oracle.build()
-    w, lres = workload_for(args.workload, args.seed, args.layers_resident)
+    w, lres = workload_for(args.workload, args.seed, args.layers_resident, args.kv_heads)
     lres = min(lres, 2)   # a couple of distinct layers, generated on the host
     caches = [inputs.layer_cache(w, l, device="cpu") for l in range(lres)]
     mode = oracle.ATTN if args.mode == "attn" else oracle.RAW
@@ -1020,6 +1026,9 @@ def main(argv=None):
     ap.add_argument("--workload", type=int, default=3,
                     help="1..5 (default 3: B 4 x 16-32K ragged, the Qwen-7B stack)")
     ap.add_argument("--mode", choices=["attn", "raw"], default="attn")
+    ap.add_argument("--kv-heads", type=int, default=None,
+                    help="another head layout of the workload: its query heads over this many KV heads "
+                         "(e.g. 1 for MQA)")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--layers-resident", type=int, default=None,
                     help="allocate this many layers and cycle them (workloads larger than HBM)")

@@ -232,18 +232,18 @@ int pow2_at_least(int n) {
 
 // The launches a scoring or attention call makes over the heads: passes of
 // at most score_max_kv_heads() KV heads (balanced), times passes of at most
-// 8 query heads of each group (the last one takes the rest).  f(goff, nkv,
-// hoff, Gn, first) is called once per pass.
+// `per_pass` query heads of each group (the last one takes the rest).
+// f(goff, nkv, hoff, Gn, first) is called once per pass.
 template <typename F>
-hill_status head_passes(const hill_desc* d, bool kv_split, F&& f) {
+hill_status head_passes(const hill_desc* d, bool kv_split, F&& f, int per_pass = 8) {
   const int Hkv = d->num_kv_heads, G = d->num_q_heads / d->num_kv_heads;
   const int cap_kv = score_max_kv_heads();
   const int kp = kv_split ? (Hkv + cap_kv - 1) / cap_kv : 1;
   bool first = true;
   for (int p = 0; p < kp; ++p) {
     const int g0 = (int)((int64_t)p * Hkv / kp), g1 = (int)((int64_t)(p + 1) * Hkv / kp);
-    for (int h0 = 0; h0 < G; h0 += 8) {
-      const hill_status s = f(g0, g1 - g0, h0, std::min(8, G - h0), first);
+    for (int h0 = 0; h0 < G; h0 += per_pass) {
+      const hill_status s = f(g0, g1 - g0, h0, std::min(per_pass, G - h0), first);
       if (s != HILL_OK) return s;
       first = false;
     }
@@ -296,10 +296,13 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
     a.hist0 = hist0;
     a.hist0_words = (int64_t)d->batch * select_hist_bins();
   }
-  // groups of more than 8 query heads are scored in passes over the same
-  // keys, and more than score_max_kv_heads() KV heads in passes over their
-  // own keys (RAW passes after the first add their sums); the kernel's group
-  // template is the power of two at or above the pass's heads
+  // more than score_max_kv_heads() KV heads are scored in passes over their
+  // own keys (RAW passes after the first add their sums); groups of more than
+  // 8 query heads are scored in passes over the same keys, except by the
+  // dealing kernel, which scores up to 32 query heads (four sub-groups of 8)
+  // from every key tile; the kernel's group template is the power of two at
+  // or above the pass's heads (8 for the dealing kernel)
+  const bool deal = L.score_spc > 1;
   a.Gs = G;
   hill_status s = part == kScoreNormalise ? HILL_OK : head_passes(d, true, [&](int goff, int nkv, int hoff, int Gn,
                                                                                 bool first) {
@@ -313,11 +316,10 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
     // later KV-head pass stores into rows no pass has written yet
     a.raw_add = kvh ? (hoff > 0 ? 1 : 0) : (first ? 0 : 1);
     // the dealing kernel exists for the group template 8 (it is chosen for
-    // groups of 5 or more heads, whose passes all fit it)
-    const bool deal = L.score_spc > 1;
+    // groups of 5 or more heads)
     return from_cuda(
         counted(launch_score(a, d->dtype, deal ? 8 : pow2_at_least(Gn), raw, f8, deal, L.score_grid, st), 1));
-  });
+  }, deal ? 4 * 8 : 8);
   if (s != HILL_OK || raw || part == kScoreStream) return s;
   FinalizeArgs f{};
   f.logits = a.logits;

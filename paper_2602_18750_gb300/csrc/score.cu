@@ -164,6 +164,16 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
   const int g0 = a.goff + (DEAL ? warp % a.nkv : warp);
   const int ng = DEAL ? (warp < W * a.nkv ? 1 : 0) : (a.nkv - warp + kNW - 1) / kNW;
   const int it0 = (DEAL && ng == 0) ? it_hi : it_lo + sub;   // this warp's first item
+  // With DEAL a warp holds one KV head, and the query heads of its group in
+  // up to kMaxNg sub-groups of 8 (a launch covers up to 32 heads per KV head):
+  // each K tile is read once and scored for every sub-group, so groups larger
+  // than 8 stream their keys once.  Fragment/statistics slot q of a warp is
+  // its q-th KV head (no DEAL) or its q-th sub-group (DEAL).
+  const int nsub = DEAL ? (a.Gn + 7) / 8 : 1;
+  auto head0_of = [&](int q) {   // first query head of slot q
+    return (DEAL ? g0 : g0 + q * kNW) * a.Gs + a.hoff + (DEAL ? 8 * q : 0);
+  };
+  auto gn_of = [&](int q) { return DEAL ? min(8, a.Gn - 8 * q) : Gn; };   // heads of slot q
 
   const uint64_t pol = l2_evict_first_policy();
   // the logits stay in L2 until the normalisation reads (and discards) them
@@ -264,9 +274,8 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
   auto load_q = [&](int b) {
 #pragma unroll
     for (int r = 0; r < kMaxNg; ++r) {
-      const bool has = r < ng && grp < Gn;
-      const int64_t row =
-          has ? (int64_t)b * a.q_sb + (int64_t)((g0 + r * kNW) * a.Gs + a.hoff + grp) * a.q_sh : 0;
+      const bool has = (DEAL ? (ng > 0 && r < nsub) : r < ng) && grp < gn_of(r);
+      const int64_t row = has ? (int64_t)b * a.q_sb + (int64_t)(head0_of(r) + grp) * a.q_sh : 0;
       if constexpr (F8) {
         const auto* qh = static_cast<const uint16_t*>(a.q) + row;
         float v[4][8];
@@ -322,8 +331,7 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
   auto flush = [&]() {
 #pragma unroll
     for (int r = 0; r < kMaxNg; ++r) {
-      if (r >= ng) break;
-      const int g = g0 + r * kNW;
+      if (DEAL ? (ng == 0 || r >= nsub) : r >= ng) break;
 #pragma unroll
       for (int c = 0; c < kCols; ++c) {
         float m = st_m[r][c], l = st_l[r][c];
@@ -336,8 +344,8 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
           m = mn;
         }
         const int hl = 2 * tig + c;
-        if (grp == 0 && hl < Gn)
-          a.partials[((int64_t)cur_b * a.nslot + cur_slot) * H + g * a.Gs + a.hoff + hl] = make_float2(m, l);
+        if (grp == 0 && hl < gn_of(r))
+          a.partials[((int64_t)cur_b * a.nslot + cur_slot) * H + head0_of(r) + hl] = make_float2(m, l);
       }
     }
   };
@@ -354,11 +362,14 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
         if (tstart[b_next + 1] == tstart[b_next]) continue;   // empty: no slots
         const int slot = ((int)blockIdx.x - tstart[b_next] / per) * W + sub;
 #pragma unroll
-        for (int c = 0; c < kCols; ++c) {
-          const int hl = 2 * tig + c;
-          if (grp == 0 && hl < Gn)
-            a.partials[((int64_t)b_next * a.nslot + slot) * H + g0 * a.Gs + a.hoff + hl] =
-                make_float2(-INFINITY, 0.f);
+        for (int q = 0; q < kMaxNg; ++q) {
+          if (q >= nsub) break;
+#pragma unroll
+          for (int c = 0; c < kCols; ++c) {
+            const int hl = 2 * tig + c;
+            if (grp == 0 && hl < gn_of(q))
+              a.partials[((int64_t)b_next * a.nslot + slot) * H + head0_of(q) + hl] = make_float2(-INFINITY, 0.f);
+          }
         }
       }
     }
@@ -383,10 +394,11 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
       cur_slot = ((int)blockIdx.x - tstart[b] / per) * W + sub;
     }
 
+    constexpr int kStagesPerItem = DEAL ? 1 : kMaxNg;   // (at most; ng of them)
 #pragma unroll
-    for (int r = 0; r < kMaxNg; ++r) {
+    for (int r = 0; r < kStagesPerItem; ++r) {
       if (r >= ng || !ok) break;
-      const int g = g0 + r * kNW;
+      const int g = DEAL ? g0 : g0 + r * kNW;
       // every lane waits; the warp goes on only if all of them saw the phase
       // complete, so it takes the same path and its shuffles stay converged
       if (!__all_sync(0xffffffffu, mbar_wait(bar0 + cs * 8, cph, a.err))) {
@@ -432,6 +444,15 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
         advance(pc);
       }
 
+      // the tile is scored for each fragment slot q: this stage's KV head
+      // (no DEAL), or every query sub-group of the warp's KV head (DEAL)
+      constexpr int kSlotsPerStage = DEAL ? kMaxNg : 1;
+#pragma unroll
+      for (int qs = 0; qs < kSlotsPerStage; ++qs) {
+      if (DEAL && qs >= nsub) break;
+      const int q = DEAL ? qs : r;
+      const int hq0 = head0_of(q);    // first query head of the slot
+      const int gnq = gn_of(q);       // its heads
       float acc[2][4];
 #pragma unroll
       for (int mb = 0; mb < 2; ++mb)
@@ -441,14 +462,14 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
       for (int kb = 0; kb < kKB; ++kb)
 #pragma unroll
         for (int mb = 0; mb < 2; ++mb) {
-          if constexpr (F8) mma_16832_e4m3(acc[mb], af[mb][kb], bq[r][kb][0], bq[r][kb][1]);
-          else mma_16816<DT>(acc[mb], af[mb][kb], bq[r][kb][0], bq[r][kb][1]);
+          if constexpr (F8) mma_16832_e4m3(acc[mb], af[mb][kb], bq[q][kb][0], bq[q][kb][1]);
+          else mma_16816<DT>(acc[mb], af[mb][kb], bq[q][kb][0], bq[q][kb][1]);
         }
       if constexpr (F8) {   // back to the key and query scales
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-          acc[u >> 1][(u & 1) * 2] *= sqA[r] * ksc[u];
-          acc[u >> 1][(u & 1) * 2 + 1] *= sqB[r] * ksc[u];
+          acc[u >> 1][(u & 1) * 2] *= sqA[q] * ksc[u];
+          acc[u >> 1][(u & 1) * 2 + 1] *= sqB[q] * ksc[u];
         }
       }
 
@@ -468,7 +489,8 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
             if (tig == 0 && t < nv) {
               const int64_t o = ((int64_t)b * Hkv + g) * cap + j0 + t;
               const float val = v * kInvSqrtD;
-              if (a.scores) a.scores[o] = a.raw_add ? a.scores[o] + val : val;
+              // later sub-groups of the same KV head add to the first one's sum
+              if (a.scores) a.scores[o] = (a.raw_add || qs > 0) ? a.scores[o] + val : val;
               if (a.accum) a.accum[o] += val;
             }
           } else {
@@ -476,7 +498,7 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
           }
         }
       } else {
-        float* lg = a.logits + ((int64_t)b * H + g * a.Gs + a.hoff) * a.lstride + j0;
+        float* lg = a.logits + ((int64_t)b * H + hq0) * a.lstride + j0;
 #pragma unroll
         for (int c = 0; c < kCols; ++c) {
           const int hl = 2 * tig + c;
@@ -486,14 +508,15 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
             const int mb = u >> 1, e = (u & 1) * 2 + c;
             const int t = mb * 16 + grp + (u & 1) * 8;
             z[u] = t < nv ? acc[mb][e] * kLog2eInvSqrtD : -INFINITY;
-            if (t < nv && hl < Gn) st_global_hint(lg + (int64_t)hl * a.lstride + t, z[u], pol_keep);
+            if (t < nv && hl < gnq) st_global_hint(lg + (int64_t)hl * a.lstride + t, z[u], pol_keep);
           }
-          const float mn = fmaxf(st_m[r][c], fmaxf(fmaxf(z[0], z[1]), fmaxf(z[2], z[3])));
-          st_l[r][c] = st_l[r][c] * ex2(st_m[r][c] - mn) +
+          const float mn = fmaxf(st_m[q][c], fmaxf(fmaxf(z[0], z[1]), fmaxf(z[2], z[3])));
+          st_l[q][c] = st_l[q][c] * ex2(st_m[q][c] - mn) +
                        ((ex2(z[0] - mn) + ex2(z[1] - mn)) + (ex2(z[2] - mn) + ex2(z[3] - mn)));
-          st_m[r][c] = mn;
+          st_m[q][c] = mn;
         }
       }
+      }   // fragment slots
     }
     if (RAW && !a.kvh) {
       // sum over the warps holding the item's heads -- all kNW (W = 1), or
