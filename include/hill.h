@@ -191,8 +191,9 @@ hill_status hill_evict_step_bkp(const hill_desc* desc, const void* q, const void
  * stream than begin, after an event recorded behind begin.  The workspace
  * belongs to the step from begin until end has completed: a pipeline over
  * layers rotates n >= 2 workspaces and issues begin of layer l + n only after
- * end of layer l (three let the K stream run two layers ahead of the
- * selection).  The scoring kernel of begin takes four fifths of the SMs, so
+ * end of layer l.  One workspace per layer leaves the K stream without any
+ * wait inside a decode step (fastest); two or three bound the memory.  The
+ * scoring kernel of begin takes four fifths of the SMs, so
  * that end's kernels have room beside it.  Results equal those of
  * hill_evict_step_bkp without attention, the ATTN scores within rounding (the
  * smaller scoring grid and the two-kernel normalisation combine the softmax

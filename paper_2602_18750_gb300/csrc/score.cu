@@ -243,7 +243,10 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
     }
   }
   pdl_wait();
-  pdl_launch_dependents();
+  // No early trigger: a dependent launches as these CTAs exit.  An early one
+  // would let the next layer's scoring grid (the next launch in this stream)
+  // take the SMs this grid leaves free for the normalisation and selection
+  // running beside it on another stream.
   if (a.hist0) {   // this CTA's share of the leading-digit histogram, zeroed for the normalisation
     const int64_t hper = (a.hist0_words + gridDim.x - 1) / gridDim.x;
     const int64_t w0 = min((int64_t)blockIdx.x * hper, a.hist0_words);

@@ -294,8 +294,8 @@ def _pipelined_layers(H, w, layers, mode, form, graph=False, nws=3):
 @pytest.mark.parametrize("n,mode", [(3, ATTN), (4, ATTN), (4, RAW)])
 def test_two_stream_pipeline_full_size(H, oracle_mod, n, mode):
     """Five layers of the 32K ragged (B 4) and 128K GQA (B 1) workloads: the
-    pipelined begin / end on two streams (two and three rotating workspaces,
-    eagerly and captured in a CUDA graph) gives the split calls' scores and
+    pipelined begin / end on two streams (two and three rotating workspaces
+    and one per layer, eagerly and captured in a CUDA graph) gives the split calls' scores and
     selections bit for bit; those agree with the serial fused step within
     the tolerance, and its selections are exact on their own keys."""
     w = inputs.config(n)
@@ -303,7 +303,7 @@ def test_two_stream_pipeline_full_size(H, oracle_mod, n, mode):
     lens, k = w.lens_at(w.steps - 1), w.budget_at(w.steps - 1)
     a = _pipelined_layers(H, w, layers, mode, "split")
     for graph in (False, True):
-        for nws in (2, 3):
+        for nws in (2, 3, layers):
             b = _pipelined_layers(H, w, layers, mode, "piped", graph, nws)
             for l in range(layers):
                 for bb, m in enumerate(lens):
