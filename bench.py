@@ -176,12 +176,12 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- schedules
-def pipelined_form(f8: bool, mode: int, accumulate: bool, lres: int) -> str:
-    """The layer-pipelined form of a workload.  The E4M3 scoring has no split
-    form; RAW scoring adds to the running importance inside the K stream, so
-    with one resident layer the next layer's stream would race the selection
-    of the previous one on the same running sums."""
-    if f8 or (accumulate and mode == 1 and lres < 2):
+def pipelined_form(mode: int, accumulate: bool, lres: int) -> str:
+    """The layer-pipelined form of a workload (the E4M3 scoring included).
+    RAW scoring adds to the running importance inside the K stream, so with
+    one resident layer the next layer's stream would race the selection of the
+    previous one on the same running sums."""
+    if accumulate and mode == 1 and lres < 2:
         return "attn-overlap"
     return "split"
 
@@ -443,8 +443,14 @@ def run_ours(args):
 
     def begin(t, l, st, wi):
         r = l % lres
-        hill.hill_evict_step_begin(desc, q_all[t, l], Kall[r], lens_all[t], max_k, mode,
-                                   accum[r] if accum is not None else None, scores[l], wss[wi], st)
+        acc = accum[r] if accum is not None else None
+        if f8:
+            hill.hill_quantize_k(desc, Kall[r], new_row[t], lens_all[t], 1, k8_all[r], ks_all[r], st)
+            hill.hill_evict_step_begin_f8(desc, q_all[t, l], k8_all[r], ks_all[r], lens_all[t], max_k, mode, acc,
+                                          scores[l], wss[wi], st)
+        else:
+            hill.hill_evict_step_begin(desc, q_all[t, l], Kall[r], lens_all[t], max_k, mode, acc, scores[l], wss[wi],
+                                       st)
 
     def end(t, l, st, wi):
         r = l % lres
@@ -460,7 +466,7 @@ def run_ours(args):
     side, att = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
     wss = [ws] + [hill.alloc_workspace(desc, mode, max_k, dev) for _ in range(SPLIT_WORKSPACES - 1)]   # evaluation
     wsa = [hill.alloc_workspace(desc, mode, max_k, dev) for _ in range(2)]   # attention
-    piped = pipelined_form(f8, mode, w.accumulate, lres)
+    piped = pipelined_form(mode, w.accumulate, lres)
     form = "serial" if args.serial else piped
     other = piped if args.serial else "serial"
 
@@ -677,7 +683,7 @@ def measure_workload(args, w, hill, dev, world, mode, full_step=False, layers_re
 
     tokens = sum(L * sum(w.lens_at(t)) for t in order)
     peak, _ = measured_peaks()
-    piped = pipelined_form(False, mode, w.accumulate, lres)
+    piped = pipelined_form(mode, w.accumulate, lres)
     runs = [(piped, False), ("serial", False)] + ([(piped, True)] if full_step else [])
     res = {}
     for frm, with_attn in dict.fromkeys(runs):

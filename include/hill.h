@@ -193,8 +193,8 @@ hill_status hill_evict_step_bkp(const hill_desc* desc, const void* q, const void
  * layers rotates n >= 2 workspaces and issues begin of layer l + n only after
  * end of layer l.  One workspace per layer leaves the K stream without any
  * wait inside a decode step (fastest); two or three bound the memory.  The
- * scoring kernel of begin takes four fifths of the SMs, so
- * that end's kernels have room beside it.  Results equal those of
+ * scoring kernel of begin takes 17/20 of the SMs, so that end's kernels have
+ * room beside it.  Results equal those of
  * hill_evict_step_bkp without attention, the ATTN scores within rounding (the
  * smaller scoring grid and the two-kernel normalisation combine the softmax
  * partials in another order); the selection follows the same rule on the
@@ -203,6 +203,12 @@ hill_status hill_evict_step_bkp(const hill_desc* desc, const void* q, const void
 hill_status hill_evict_step_begin(const hill_desc* desc, const void* q, const void* k_cache,
                                   const int32_t* lens, int32_t max_k, hill_score_mode mode, float* accum,
                                   float* scores, void* ws, size_t ws_bytes, void* stream);
+/* hill_evict_step_begin with the keys scored from their E4M3 shadow (k8,
+ * kscale as in hill_score_f8 below): the split form of hill_evict_step_f8's
+ * evaluation, completed by hill_evict_step_end in the same way. */
+hill_status hill_evict_step_begin_f8(const hill_desc* desc, const void* q, const uint8_t* k8, const float* kscale,
+                                     const int32_t* lens, int32_t max_k, hill_score_mode mode, float* accum,
+                                     float* scores, void* ws, size_t ws_bytes, void* stream);
 hill_status hill_evict_step_end(const hill_desc* desc, const int32_t* lens, const int32_t* k, int32_t recent,
                                 int32_t max_k, hill_score_mode mode, float* accum, float* scores,
                                 int32_t* idx, int32_t* count, uint16_t* hits, void* ws, size_t ws_bytes,

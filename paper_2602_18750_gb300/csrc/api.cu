@@ -165,13 +165,17 @@ struct Layout {
 };
 
 // The scoring kernel's grid: one CTA per SM, or in the split step
-// (split_grid) four fifths of them, so that the normalisation and selection of
-// the previous layer find whole SMs beside the K stream (the stream itself is
-// bound by HBM, not by the number of SMs streaming).
+// (split_grid) 17/20 of them, so that the normalisation and selection of the
+// previous layer find whole SMs beside the K stream.  Measured on the 32K and
+// 128K workloads: the 16-bit stream, bound by HBM, is as fast on 4/5 or 17/20
+// of the SMs and slower on 9/10; the E4M3 stream, bound by the latency of its
+// per-tile chain, gains with every SM (4/5: 80 / 48 us per layer, 17/20: 76 /
+// 45, 9/10: 74 / 45).  One fraction for both, since end() must find the
+// partial slots that begin() wrote without knowing the key format.
 int score_grid_for(const hill_desc* d, int sms, bool split_grid = false) {
   const int T = score_tile_tokens();
   const long long items = (long long)d->batch * ((d->capacity + T - 1) / T);
-  long long g = split_grid ? sms * 4 / 5 : sms;
+  long long g = split_grid ? sms * 17 / 20 : sms;
   if (items < g) g = items;
   return g < 1 ? 1 : (int)g;
 }
@@ -551,14 +555,19 @@ hill_status hill_topk_select_bkp(const hill_desc* desc, const float* scores, con
                     recent, hits);
 }
 
-hill_status hill_evict_step_begin(const hill_desc* desc, const void* q, const void* k_cache, const int32_t* lens,
-                                  int32_t max_k, hill_score_mode mode, float* accum, float* scores, void* ws,
-                                  size_t ws_bytes, void* stream) {
+}  // extern "C"
+
+namespace {
+// The K stream of the split step, from the 16-bit cache (kscale NULL) or from
+// its E4M3 shadow (k = the codes, kscale = the row scales).
+hill_status evict_step_begin(const hill_desc* desc, const void* q, const void* k, const float* kscale,
+                             const int32_t* lens, int32_t max_k, hill_score_mode mode, float* accum, float* scores,
+                             void* ws, size_t ws_bytes, void* stream) {
   hill_status s = check_desc(desc);
   if (s != HILL_OK) return s;
   if (mode != HILL_SCORE_ATTN && mode != HILL_SCORE_RAW) return HILL_ERR_INVALID_ARG;
-  if (max_k < 0 || !q || !k_cache || !lens) return HILL_ERR_INVALID_ARG;
-  if (!aligned16(q) || !aligned16(k_cache)) return HILL_ERR_INVALID_ARG;
+  if (max_k < 0 || !q || !k || !lens) return HILL_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || (kscale && !aligned16(kscale))) return HILL_ERR_INVALID_ARG;
   DeviceInfo di;
   if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
   const Layout L = layout_for(desc, mode, max_k, di.sms, false, true);
@@ -566,8 +575,24 @@ hill_status hill_evict_step_begin(const hill_desc* desc, const void* q, const vo
   unsigned char* base = ws_base(ws);
   float* s_out = scores ? scores : (accum ? nullptr : reinterpret_cast<float*>(base + L.scores));
   uint32_t* hist0 = L.has_hist0 ? reinterpret_cast<uint32_t*>(base + L.hist0) : nullptr;
-  return run_score(desc, q, k_cache, lens, mode, s_out, accum, base, L, di, static_cast<cudaStream_t>(stream),
-                   hist0, 0, nullptr, false, kScoreStream);
+  return run_score(desc, q, k, lens, mode, s_out, accum, base, L, di, static_cast<cudaStream_t>(stream), hist0, 0,
+                   kscale, false, kScoreStream);
+}
+}  // namespace
+
+extern "C" {
+
+hill_status hill_evict_step_begin(const hill_desc* desc, const void* q, const void* k_cache, const int32_t* lens,
+                                  int32_t max_k, hill_score_mode mode, float* accum, float* scores, void* ws,
+                                  size_t ws_bytes, void* stream) {
+  return evict_step_begin(desc, q, k_cache, nullptr, lens, max_k, mode, accum, scores, ws, ws_bytes, stream);
+}
+
+hill_status hill_evict_step_begin_f8(const hill_desc* desc, const void* q, const uint8_t* k8, const float* kscale,
+                                     const int32_t* lens, int32_t max_k, hill_score_mode mode, float* accum,
+                                     float* scores, void* ws, size_t ws_bytes, void* stream) {
+  if (!k8 || !kscale) return HILL_ERR_INVALID_ARG;
+  return evict_step_begin(desc, q, k8, kscale, lens, max_k, mode, accum, scores, ws, ws_bytes, stream);
 }
 
 hill_status hill_evict_step_end(const hill_desc* desc, const int32_t* lens, const int32_t* k, int32_t recent,

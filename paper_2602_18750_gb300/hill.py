@@ -9,8 +9,8 @@ fails loudly if the library has not been built.
 Names follow the C ABI: :func:`hill_score`, :func:`hill_topk_select`,
 :func:`hill_gather_sparse_attn`, :func:`hill_evict_step`, :func:`hill_topk_select_bkp`,
 :func:`hill_evict_step_bkp`, :func:`hill_quantize_k`, :func:`hill_score_f8`, :func:`hill_evict_step_f8`,
-:func:`hill_evict_step_kvh`, :func:`hill_evict_step_begin`, :func:`hill_evict_step_end`,
-:func:`hill_workspace_bytes`, :func:`hill_sync_status`.
+:func:`hill_evict_step_kvh`, :func:`hill_evict_step_begin`, :func:`hill_evict_step_begin_f8`,
+:func:`hill_evict_step_end`, :func:`hill_workspace_bytes`, :func:`hill_sync_status`.
 """
 from __future__ import annotations
 
@@ -77,6 +77,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_quantize_k.argtypes = [D, P, P, P, I32, P, P, P]
     lib.hill_evict_step_kvh.argtypes = [D, P, P, P, P, P, I32, I32, P, P, P, P, P, P, SZ, P]
     lib.hill_evict_step_begin.argtypes = [D, P, P, P, I32, I32, P, P, P, SZ, P]
+    lib.hill_evict_step_begin_f8.argtypes = [D, P, P, P, P, I32, I32, P, P, P, SZ, P]
     lib.hill_evict_step_end.argtypes = [D, P, P, I32, I32, I32, P, P, P, P, P, P, SZ, P]
     lib.hill_selftest_wait.argtypes = [ctypes.c_uint32, P]
     lib.hill_score_f8.argtypes = [D, P, P, P, P, I32, P, P, P, SZ, P]
@@ -90,8 +91,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.hill_kernel_launches.restype = ctypes.c_uint64
     for name in ("hill_score", "hill_topk_select", "hill_gather_sparse_attn", "hill_evict_step",
                  "hill_topk_select_bkp", "hill_evict_step_bkp", "hill_quantize_k", "hill_score_f8",
-                 "hill_evict_step_f8", "hill_evict_step_kvh", "hill_evict_step_begin", "hill_evict_step_end",
-                 "hill_selftest_wait", "hill_sync_status"):
+                 "hill_evict_step_f8", "hill_evict_step_kvh", "hill_evict_step_begin", "hill_evict_step_begin_f8",
+                 "hill_evict_step_end", "hill_selftest_wait", "hill_sync_status"):
         getattr(lib, name).restype = I32
     _lib = lib
     return lib
@@ -220,6 +221,14 @@ def hill_evict_step_begin(desc, q, k_cache, lens, max_k, mode, accum, scores, ws
     _check(load().hill_evict_step_begin(ctypes.byref(desc), _ptr(q), _ptr(k_cache), _ptr(lens), int(max_k),
                                         int(mode), _ptr(accum), _ptr(scores), wp, wn, _stream(stream)),
            "hill_evict_step_begin")
+
+
+def hill_evict_step_begin_f8(desc, q, k8, kscale, lens, max_k, mode, accum, scores, ws, stream=None) -> None:
+    """First half of the split step from the E4M3 key shadow."""
+    wp, wn = _ws(ws)
+    _check(load().hill_evict_step_begin_f8(ctypes.byref(desc), _ptr(q), _ptr(k8), _ptr(kscale), _ptr(lens),
+                                           int(max_k), int(mode), _ptr(accum), _ptr(scores), wp, wn,
+                                           _stream(stream)), "hill_evict_step_begin_f8")
 
 
 def hill_evict_step_end(desc, lens, k, max_k, mode, accum, scores, idx, count, ws, recent=0, hits=None,

@@ -8,8 +8,9 @@ the building block of the layer-pipelined evaluation (Sec. 4.3):
   windows and hit tables, and the budget edge cases;
 * the split step against the oracle (scores, selection by the gap rule) and
   against the fused hill_evict_step (RAW: bit for bit; ATTN: scores within
-  the tolerance, since the split step's scoring grid -- four fifths of the
-  SMs -- combines the softmax partials in another order);
+  the tolerance, since the split step's scoring grid -- 17/20 of the SMs --
+  combines the softmax partials in another order), from the 16-bit
+  keys and from their E4M3 shadow (begin_f8 against hill_evict_step_f8);
 * two streams and rotating workspaces over the layers of the 32K and 128K
   workloads, eagerly and in a CUDA graph, bit for bit against the same split
   calls issued one after another on one stream, and within the tolerance of
@@ -173,6 +174,46 @@ def test_split_step_matches_oracle_and_fused(H, oracle_mod, mode, shape):
         for b, n in enumerate(lens):
             assert torch.equal(scores[b, :n], ev.scores[b, :n])
         assert torch.equal(idx, ev.idx) and torch.equal(cnt, ev.count)
+
+
+@pytest.mark.parametrize("mode", [ATTN, RAW])
+@pytest.mark.parametrize("shape", SHAPES, ids=lambda s: f"B{s[0]}H{s[1]}kv{s[2]}cap{s[3]}")
+def test_split_step_f8_matches_oracle_and_fused(H, oracle_mod, mode, shape):
+    """hill_evict_step_begin_f8 + end on the E4M3 shadow: scores against the
+    oracle's logits on the 8-bit operands, the selection exact on its own
+    keys, and against the fused hill_evict_step_f8 (RAW bit for bit, ATTN
+    within the tolerance)."""
+    B, Hq, Hkv, cap, lens, k = shape
+    q, K, V, lens_t = inputs.random_case(B, Hq, Hkv, 128, cap, lens, dtype=torch.bfloat16, seed=cap + 3 * Hq,
+                                         kind="zipf" if Hq == Hkv else "normal")
+    q, K, V, lens_t = q.cuda(), K.cuda(), V.cuda(), lens_t.cuda()
+    max_k = max(max(k), 1)
+    desc = H.make_desc(q, K, V)
+    k8, ks = H.alloc_shadow(desc)
+    H.hill_quantize_k(desc, K, _i32([0] * B), lens_t, cap, k8, ks)
+    ws = H.alloc_workspace(desc, mode, max_k)
+    scores = torch.full((B, cap), float("nan"), device="cuda")
+    idx = torch.empty(B, max_k, dtype=torch.int32, device="cuda")
+    cnt = torch.empty(B, dtype=torch.int32, device="cuda")
+    H.hill_evict_step_begin_f8(desc, q, k8, ks, lens_t, max_k, mode, None, scores, ws)
+    H.hill_evict_step_end(desc, lens_t, _i32(k), max_k, mode, None, scores, idx, cnt, ws)
+    H.hill_sync_status()
+    codes, scale = oracle_mod.quantize_rows(K.cpu())
+    s_ref = oracle_mod.scores(mode, oracle_mod.logits_q8(q.cpu(), codes, scale, lens), lens)
+    check_scores(scores.cpu().numpy(), s_ref, lens)
+    check_selection(idx.cpu().numpy(), cnt.cpu().numpy(), s_ref, lens, k, max_k)
+    idx_o, cnt_o, _ = oracle_mod.topk(scores.cpu().numpy().astype(np.float64), lens, k, max_k)
+    assert np.array_equal(idx.cpu().numpy(), idx_o) and np.array_equal(cnt.cpu().numpy(), cnt_o)
+    s_f = torch.full((B, cap), float("nan"), device="cuda")
+    idx_f = torch.empty_like(idx)
+    cnt_f = torch.empty_like(cnt)
+    H.hill_evict_step_f8(desc, q, k8, ks, K, V, lens_t, _i32(k), max_k, mode, None, s_f, idx_f, cnt_f, None, ws)
+    H.hill_sync_status()
+    check_scores(scores.cpu().numpy(), s_f.cpu().numpy().astype(np.float64), lens, what="split vs fused")
+    if mode == RAW:
+        for b, n in enumerate(lens):
+            assert torch.equal(scores[b, :n], s_f[b, :n])
+        assert torch.equal(idx, idx_f) and torch.equal(cnt, cnt_f)
 
 
 @pytest.mark.parametrize("mode", [ATTN, RAW])
