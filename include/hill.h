@@ -45,10 +45,12 @@
  *   touched.  k[b] is clamped to [0, lens[b]].
  * - Supported: head_dim 128; any H and Hkv with H a multiple of Hkv (MHA,
  *   GQA with any group size G = H / Hkv, MQA); B <= 512; fp16 or bf16 q/K/V.
- *   Groups of more than 8 query heads are scored and attended in passes of at
- *   most 8 over the same KV rows, and more than 32 KV heads are scored in
- *   passes of at most 32 (e.g. 40 KV heads: two passes of 20), each pass
- *   streaming only its own heads' keys.
+ *   Groups of more than 8 query heads are scored in passes of at most 8 over
+ *   the same keys, except with at most 4 KV heads (MQA-like), where one pass
+ *   scores up to 32 query heads of each KV head from every key tile; the
+ *   attention takes up to 16 query heads per pass over the gathered rows.
+ *   More than 32 KV heads are scored in passes of at most 32 (e.g. 40 KV
+ *   heads: two passes of 20), each pass streaming only its own heads' keys.
  */
 #ifndef HILL_H_
 #define HILL_H_

@@ -402,7 +402,7 @@ hill_status run_attn(const hill_desc* d, const void* q, const void* k, const voi
   a.splits = L.splits;
   a.kvh = kvh ? 1 : 0;
   a.err = di.err;
-  // G > 8 query heads per KV head: passes of at most 8 heads over the same
+  // G > 16 query heads per KV head: passes of at most 16 heads over the same
   // selected rows, then one merge of the split partials over all heads
   const int G = d->num_q_heads / d->num_kv_heads;
   a.Gs = G;
@@ -412,7 +412,7 @@ hill_status run_attn(const hill_desc* d, const void* q, const void* k, const voi
     const bool last = hoff + Gn == G;
     return from_cuda(
         counted(launch_sparse_attn(a, d->dtype, pow2_at_least(Gn), L.attn_grid, last, st), last ? 2 : 1));
-  });
+  }, 16);
 }
 
 }  // namespace

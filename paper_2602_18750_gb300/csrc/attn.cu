@@ -26,7 +26,10 @@
 // V^T . P^T: V rows read with transposed ldmatrix form A (16 dims x 16
 // tokens), and the weights P -- already laid out as a B fragment by the S
 // accumulators -- enter as a 16-bit high part plus its 16-bit residual, so
-// every instruction covers 8 heads x 16 dims.  When a warp's segment holds
+// every instruction covers 8 heads x 16 dims.  A group of 9 to 16 heads fills
+// all 16 rows of A (two row blocks of 8 heads, each with its own softmax state
+// and O^T accumulators), so the rows gathered once serve 16 heads; larger
+// groups run in passes of 16.  When a warp's segment holds
 // all batches of a (b, g) it writes the output; otherwise it writes a partial
 // (max, sum, o) that hill_attn_combine_kernel merges.
 #include <type_traits>
@@ -204,33 +207,42 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
   advance(pl);
 
   // mma.sync fragments: grp = lane/4, tig = lane%4.  S accumulators: row grp
-  // = query head grp of the group (rows >= Gn and 8..15 are zero; Gn = G
-  // unless G is 4 or 8 and the group has 3, or 5 to 7 heads), columns =
-  // tokens nb*8 + 2*tig + {0,1}.  O^T accumulators: rows = dims db*16 + grp
-  // (+8), columns = heads 2*tig, 2*tig + 1.
+  // (+8 with 16 heads: row block rb = 1) = query head grp (+8) of the group
+  // (rows >= Gn are zero, and rows 8..15 when G <= 8; Gn = G unless the
+  // group has fewer heads than the power-of-two template), columns = tokens
+  // nb*8 + 2*tig + {0,1}.  O^T accumulators, one set per row block: rows =
+  // dims db*16 + grp (+8), columns = heads 8*rb + 2*tig, 8*rb + 2*tig + 1.
+  constexpr int kRB = G > 8 ? 2 : 1;          // row blocks of 8 heads
   const int grp = lane >> 2, tig = lane & 3;
   const int Gn = G <= 2 ? G : a.Gn;
-  const bool head_ok = grp < Gn;
-  const int hA = 2 * tig, hB = 2 * tig + 1;   // heads of this lane's O^T columns
-  float m_run = -INFINITY, l_run = 0.f;       // softmax state of head grp (base 2)
-  float oacc[8][4];
-  uint32_t qa[8][2];                          // q rows of the group as A fragments
+  bool head_ok[kRB];
+#pragma unroll
+  for (int rb = 0; rb < kRB; ++rb) head_ok[rb] = grp + 8 * rb < Gn;
+  const int hA = 2 * tig, hB = 2 * tig + 1;   // heads of this lane's O^T columns (in a row block)
+  float m_run[kRB], l_run[kRB];               // softmax state of head grp + 8*rb (base 2)
+  float oacc[kRB][8][4];
+  uint32_t qa[kRB][8][2];                     // q rows of the group as A fragments
   int cb = -1, cg = -1, cu = -1;              // the (b, g) being accumulated and its unit
   const int per = (total + nwarps - 1) / nwarps;
 
   auto reset = [&](int b, int g) {
-    m_run = -INFINITY;
-    l_run = 0.f;
-#pragma unroll
-    for (int db = 0; db < 8; ++db)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) oacc[db][e] = 0.f;
     const auto* q32 = static_cast<const uint32_t*>(a.q);
-    const int64_t row = head_ok ? ((int64_t)b * a.q_sb + (int64_t)(g * a.Gs + a.hoff + grp) * a.q_sh) / 2 : 0;
 #pragma unroll
-    for (int kb = 0; kb < 8; ++kb) {
-      qa[kb][0] = head_ok ? __ldg(q32 + row + kb * 8 + tig) : 0u;
-      qa[kb][1] = head_ok ? __ldg(q32 + row + kb * 8 + 4 + tig) : 0u;
+    for (int rb = 0; rb < kRB; ++rb) {
+      m_run[rb] = -INFINITY;
+      l_run[rb] = 0.f;
+#pragma unroll
+      for (int db = 0; db < 8; ++db)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) oacc[rb][db][e] = 0.f;
+      const bool ok = head_ok[rb];
+      const int64_t row =
+          ok ? ((int64_t)b * a.q_sb + (int64_t)(g * a.Gs + a.hoff + 8 * rb + grp) * a.q_sh) / 2 : 0;
+#pragma unroll
+      for (int kb = 0; kb < 8; ++kb) {
+        qa[rb][kb][0] = ok ? __ldg(q32 + row + kb * 8 + tig) : 0u;
+        qa[rb][kb][1] = ok ? __ldg(q32 + row + kb * 8 + 4 + tig) : 0u;
+      }
     }
   };
 
@@ -241,33 +253,38 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
     const int firstb = s_bstart[cu] + (a.kvh ? 0 : cg * nb_);   // first batch of (cb, cg) in the list
     const bool whole = firstb / per == (firstb + nb_ - 1) / per;   // one segment holds it all
     const int seg = gw - firstb / per;
-    // (max, sum) of the heads in this lane's O^T columns
-    const float mA = __shfl_sync(0xffffffffu, m_run, 8 * tig), lA = __shfl_sync(0xffffffffu, l_run, 8 * tig);
-    const float mB = __shfl_sync(0xffffffffu, m_run, 8 * tig + 4), lB = __shfl_sync(0xffffffffu, l_run, 8 * tig + 4);
 #pragma unroll
-    for (int c = 0; c < 2; ++c) {
-      const int hl = c ? hB : hA;
-      if (hl >= Gn) continue;
-      const float m = c ? mB : mA, l = c ? lB : lA;
-      const int h = cg * a.Gs + a.hoff + hl;
-      if (whole) {
-        float* op = a.out + ((int64_t)cb * a.H + h) * kHeadDim + grp;
-        const float inv = l > 0.f ? 1.f / l : 0.f;
+    for (int rb = 0; rb < kRB; ++rb) {
+      // (max, sum) of the heads in this lane's O^T columns of row block rb
+      const float mA = __shfl_sync(0xffffffffu, m_run[rb], 8 * tig);
+      const float lA = __shfl_sync(0xffffffffu, l_run[rb], 8 * tig);
+      const float mB = __shfl_sync(0xffffffffu, m_run[rb], 8 * tig + 4);
+      const float lB = __shfl_sync(0xffffffffu, l_run[rb], 8 * tig + 4);
 #pragma unroll
-        for (int db = 0; db < 8; ++db) {
-          op[db * 16] = oacc[db][c] * inv;
-          op[db * 16 + 8] = oacc[db][2 + c] * inv;
-        }
-      } else {
-        float* pp = a.part + (((int64_t)cb * a.H + h) * a.splits + seg) * (2 + kHeadDim);
-        if (grp == 0) {
-          pp[0] = m;
-          pp[1] = l;
-        }
+      for (int c = 0; c < 2; ++c) {
+        const int hl = 8 * rb + (c ? hB : hA);
+        if (hl >= Gn) continue;
+        const float m = c ? mB : mA, l = c ? lB : lA;
+        const int h = cg * a.Gs + a.hoff + hl;
+        if (whole) {
+          float* op = a.out + ((int64_t)cb * a.H + h) * kHeadDim + grp;
+          const float inv = l > 0.f ? 1.f / l : 0.f;
 #pragma unroll
-        for (int db = 0; db < 8; ++db) {
-          pp[2 + db * 16 + grp] = oacc[db][c];
-          pp[2 + db * 16 + 8 + grp] = oacc[db][2 + c];
+          for (int db = 0; db < 8; ++db) {
+            op[db * 16] = oacc[rb][db][c] * inv;
+            op[db * 16 + 8] = oacc[rb][db][2 + c] * inv;
+          }
+        } else {
+          float* pp = a.part + (((int64_t)cb * a.H + h) * a.splits + seg) * (2 + kHeadDim);
+          if (grp == 0) {
+            pp[0] = m;
+            pp[1] = l;
+          }
+#pragma unroll
+          for (int db = 0; db < 8; ++db) {
+            pp[2 + db * 16 + grp] = oacc[rb][db][c];
+            pp[2 + db * 16 + 8 + grp] = oacc[rb][db][2 + c];
+          }
         }
       }
     }
@@ -299,8 +316,11 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
         const int c = 4 * kp + (lane >> 3);
         uint32_t bk[4];
         ldmatrix_x4(sk + (c >> 3) * kHalfBytes + trow * 128 + (((c & 7) ^ (trow & 7)) << 4), bk);
-        const uint32_t a0[4] = {qa[2 * kp][0], 0u, qa[2 * kp][1], 0u};
-        const uint32_t a1[4] = {qa[2 * kp + 1][0], 0u, qa[2 * kp + 1][1], 0u};
+        // rows 8..15 of A: the second row block of 16 heads, else zero
+        const uint32_t a0[4] = {qa[0][2 * kp][0], kRB > 1 ? qa[kRB - 1][2 * kp][0] : 0u, qa[0][2 * kp][1],
+                                kRB > 1 ? qa[kRB - 1][2 * kp][1] : 0u};
+        const uint32_t a1[4] = {qa[0][2 * kp + 1][0], kRB > 1 ? qa[kRB - 1][2 * kp + 1][0] : 0u,
+                                qa[0][2 * kp + 1][1], kRB > 1 ? qa[kRB - 1][2 * kp + 1][1] : 0u};
         mma_16816<DT>(sacc[nb], a0, bk[0], bk[1]);
         mma_16816<DT>(sacc[nb], a1, bk[2], bk[3]);
       }
@@ -314,57 +334,61 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
       jnext = t + 2 < t1 ? load_idx(pl) : -1;
       advance(pl);
     }
-    // online softmax of head grp over the batch's tokens nb*8 + 2*tig + {0,1}
-    float z[8];
-    float tmax = -INFINITY;
+    // online softmax of head grp (+8 for row block 1) over the batch's tokens
+    // nb*8 + 2*tig + {0,1}
+    uint32_t pb[kRB][2][2][2];   // [row block][k block][hi/lo][tokens 0-7 | 8-15 of the block]
 #pragma unroll
-    for (int nb = 0; nb < 4; ++nb)
+    for (int rb = 0; rb < kRB; ++rb) {
+      float z[8];
+      float tmax = -INFINITY;
 #pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int tkn = nb * 8 + 2 * tig + e;
-        const float v = ((vm >> tkn) & 1u) ? sacc[nb][e] * kLog2eInvSqrtD : -INFINITY;
-        z[nb * 2 + e] = v;
-        tmax = fmaxf(tmax, v);
+      for (int nb = 0; nb < 4; ++nb)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int tkn = nb * 8 + 2 * tig + e;
+          const float v = ((vm >> tkn) & 1u) ? sacc[nb][2 * rb + e] * kLog2eInvSqrtD : -INFINITY;
+          z[nb * 2 + e] = v;
+          tmax = fmaxf(tmax, v);
+        }
+      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
+      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
+      const float mn = fmaxf(m_run[rb], tmax);   // finite: every batch holds a token
+      const float corr = ex2(m_run[rb] - mn);    // 0 on the first batch
+      float p[8], psum = 0.f;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        p[u] = head_ok[rb] ? ex2(z[u] - mn) : 0.f;
+        psum += p[u];
       }
-    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
-    tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
-    const float mn = fmaxf(m_run, tmax);      // finite: every batch holds a token
-    const float corr = ex2(m_run - mn);       // 0 on the first batch
-    float p[8], psum = 0.f;
+      psum += __shfl_xor_sync(0xffffffffu, psum, 1);
+      psum += __shfl_xor_sync(0xffffffffu, psum, 2);
+      l_run[rb] = l_run[rb] * corr + psum;
+      m_run[rb] = mn;
+      // rescale O^T: columns hA, hB take the factor of their head
+      const float cA = __shfl_sync(0xffffffffu, corr, 8 * tig);
+      const float cB = __shfl_sync(0xffffffffu, corr, 8 * tig + 4);
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      p[u] = head_ok ? ex2(z[u] - mn) : 0.f;
-      psum += p[u];
+      for (int db = 0; db < 8; ++db) {
+        oacc[rb][db][0] *= cA;
+        oacc[rb][db][2] *= cA;
+        if constexpr (G > 1) {
+          oacc[rb][db][1] *= cB;
+          oacc[rb][db][3] *= cB;
+        }
+      }
+      // P as B fragments (k = token, n = head grp), split into a 16-bit high
+      // part and its 16-bit residual so the weights keep ~22 bits
+#pragma unroll
+      for (int kt = 0; kt < 2; ++kt)
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {
+          const float x = p[(2 * kt + hf) * 2], y = p[(2 * kt + hf) * 2 + 1];
+          const uint32_t hi = pack2<DT>(x, y);
+          const float2 hv = unpack2<DT>(hi);
+          pb[rb][kt][0][hf] = hi;
+          pb[rb][kt][1][hf] = pack2<DT>(x - hv.x, y - hv.y);
+        }
     }
-    psum += __shfl_xor_sync(0xffffffffu, psum, 1);
-    psum += __shfl_xor_sync(0xffffffffu, psum, 2);
-    l_run = l_run * corr + psum;
-    m_run = mn;
-    // rescale O^T: columns hA, hB take the factor of their head
-    const float cA = __shfl_sync(0xffffffffu, corr, 8 * tig);
-    const float cB = __shfl_sync(0xffffffffu, corr, 8 * tig + 4);
-#pragma unroll
-    for (int db = 0; db < 8; ++db) {
-      oacc[db][0] *= cA;
-      oacc[db][2] *= cA;
-      if constexpr (G > 1) {
-        oacc[db][1] *= cB;
-        oacc[db][3] *= cB;
-      }
-    }
-    // P as B fragments (k = token, n = head grp), split into a 16-bit high
-    // part and its 16-bit residual so the weights keep ~22 bits
-    uint32_t pb[2][2][2];   // [k block][hi/lo][tokens 0-7 | 8-15 of the block]
-#pragma unroll
-    for (int kt = 0; kt < 2; ++kt)
-#pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {
-        const float x = p[(2 * kt + hf) * 2], y = p[(2 * kt + hf) * 2 + 1];
-        const uint32_t hi = pack2<DT>(x, y);
-        const float2 hv = unpack2<DT>(hi);
-        pb[kt][0][hf] = hi;
-        pb[kt][1][hf] = pack2<DT>(x - hv.x, y - hv.y);
-      }
     // V(t) is complete once at most K(t + 1) is pending
     if (more) cp_async_wait<1>();
     else cp_async_wait<0>();
@@ -378,8 +402,11 @@ __global__ void __launch_bounds__(kAThreads, 1) hill_sparse_attn_kernel(const __
         const int c = 2 * db + ((lane >> 3) & 1);
         uint32_t av[4];
         ldmatrix_x4_trans(sv + (c >> 3) * kHalfBytes + trow * 128 + (((c & 7) ^ (trow & 7)) << 4), av);
-        mma_16816<DT>(oacc[db], av, pb[kt][0][0], pb[kt][0][1]);
-        mma_16816<DT>(oacc[db], av, pb[kt][1][0], pb[kt][1][1]);
+#pragma unroll
+        for (int rb = 0; rb < kRB; ++rb) {
+          mma_16816<DT>(oacc[rb][db], av, pb[rb][kt][0][0], pb[rb][kt][0][1]);
+          mma_16816<DT>(oacc[rb][db], av, pb[rb][kt][1][0], pb[rb][kt][1][1]);
+        }
       }
     }
     // the V region is free: fetch V(t + 1)
@@ -518,6 +545,7 @@ cudaError_t launch_attn_d(const AttnArgs& a, int G, int grid, bool combine, cuda
     case 2: return launch_attn_t<DT, 2>(a, grid, combine, st);
     case 4: return launch_attn_t<DT, 4>(a, grid, combine, st);
     case 8: return launch_attn_t<DT, 8>(a, grid, combine, st);
+    case 16: return launch_attn_t<DT, 16>(a, grid, combine, st);
   }
   return cudaErrorInvalidValue;
 }

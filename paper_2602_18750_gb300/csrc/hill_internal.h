@@ -33,9 +33,9 @@ struct ScoreArgs {
   // handles (hoff) and how many (Gn, at most the kernel's template group G,
   // the rows past Gn being zero): a launch covers heads g * Gs + hoff +
   // [0, Gn) of the KV heads g in [goff, goff + nkv).  Groups of more than 8
-  // heads are scored in passes of at most 8, and more than 32 KV heads in
-  // passes of at most 32; RAW passes after the first add to scores (raw_add)
-  // instead of storing.
+  // heads are scored in passes of at most 8 (the dealing kernel: 32), and more
+  // than 32 KV heads in passes of at most 32; RAW passes after the first add
+  // to scores (raw_add) instead of storing.
   int Gs, hoff, Gn, goff, nkv, raw_add;
   uint32_t* hist0;    // optional: zero-filled here (hist0_words words) for the normalisation to count into
   int64_t hist0_words;

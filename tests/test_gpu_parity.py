@@ -54,11 +54,14 @@ SHAPES = [
     # fewer query heads than one warp of the normalisation combines
     (2, 2, 1, 300, [300, 150], [30, 15]),
     (2, 1, 1, 257, [257, 100], [20, 100]),
-    # groups of more than 8 query heads per KV head (MQA-like), run in passes of 8
+    # groups of more than 8 query heads per KV head (MQA-like): the scoring
+    # kernel scores up to 32 from each key tile, the attention up to 16 from
+    # each gathered batch (32 = two passes of 16)
     (2, 32, 1, 700, [700, 333], [70, 33]),
     (2, 32, 2, 500, [500, 260], [50, 26]),
     # group sizes that are not powers of two (the kernels' power-of-two group
-    # templates with the extra query rows zero), and one of 12 = 8 + 4 heads
+    # templates with the extra query rows zero), and one of 12 heads (the
+    # attention's 16-head template with 4 rows zero)
     (2, 12, 4, 300, [300, 171], [30, 17]),
     (2, 28, 4, 400, [400, 95], [40, 9]),
     (1, 24, 2, 257, [257], [25]),
