@@ -810,7 +810,8 @@ def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all,
     idx_h = torch.empty_like(idx, device="cpu").pin_memory()
     cnt_h = torch.empty_like(count, device="cpu").pin_memory()
     out_h = torch.empty_like(out, device="cpu").pin_memory()
-    uniform = [len(set(p)) == 1 for p in pos]
+    pos_d = [torch.tensor(p, dtype=torch.long, device=dev) for p in pos]
+    b_d = torch.arange(B, device=dev)
     # per-layer views, made once (as an engine would hold them)
     qv = [[q_all[t, l] for l in range(L)] for t in range(S)]
     Kv, Vv = [Kall[r] for r in range(lres)], [Vall[r] for r in range(lres)]
@@ -840,13 +841,10 @@ def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all,
         issue_layers(form, L, stream, side, att, True, fused, begin, end, attn)
 
     def append(t, sk, sv):
-        if uniform[t]:
-            Kall[:, :, :, pos[t][0]].copy_(sk)
-            Vall[:, :, :, pos[t][0]].copy_(sv)
-        else:
-            for b in range(B):
-                Kall[:, b, :, pos[t][b]].copy_(sk[:, b])
-                Vall[:, b, :, pos[t][b]].copy_(sv[:, b])
+        # the new token's K/V row of every resident layer and sequence, one
+        # indexed write per cache: K[:, b, :, pos[b]] = sk[:, b] for every b
+        Kall[:, b_d, :, pos_d[t]] = sk.transpose(0, 1)
+        Vall[:, b_d, :, pos_d[t]] = sv.transpose(0, 1)
 
     res0 = (list(idx), list(count), list(out))
 
@@ -862,9 +860,12 @@ def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all,
         out_h.copy_(out, non_blocking=True)
 
     # Overlapped form (what a serving loop does): while step t computes, a copy
-    # stream brings in step t + 1's inputs and copies out step t - 1's results.
-    # Inputs are staged and results written in two alternating buffer sets,
-    # so a step's compute never touches the buffers being copied.
+    # stream brings in step t + 1's inputs -- its queries, lengths and budgets,
+    # and its new K/V rows, written into the caches at once -- and copies out
+    # step t - 1's results.  Inputs are staged and results written in two
+    # alternating buffer sets, so a step's compute never touches the buffers
+    # being copied; the new rows of step t + 1 lie at or past step t's
+    # lengths, where step t's kernels use no key or value.
     cstream = torch.cuda.Stream(device=dev)
     stage2_k = torch.empty((2,) + tuple(stage_k.shape), dtype=w.dtype, device=dev)
     stage2_v = torch.empty_like(stage2_k)
@@ -884,12 +885,12 @@ def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all,
         cstream.wait_event(cfork)
         with torch.cuda.stream(cstream):
             stage_in((t + 1) % S, 1 - par)
+            append((t + 1) % S, stage2_k[1 - par], stage2_v[1 - par])
             pi, pc, po = res[1 - par]
             idx_h.copy_(pi, non_blocking=True)
             cnt_h.copy_(pc, non_blocking=True)
             out_h.copy_(po, non_blocking=True)
         cjoin.record(cstream)
-        append(t, stage2_k[par], stage2_v[par])
         compute(t, lk2_d[par][0], lk2_d[par][1], *resv[par])
         stream.wait_event(cjoin)
 
@@ -919,6 +920,7 @@ def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all,
     # copies overlapped with the compute as above
     with torch.cuda.stream(stream):
         stage_in(0, 0)
+        append(0, stage2_k[0], stage2_v[0])
     stream.synchronize()
     graphs = {}
     for i in range(args.warmup + len(order)):
@@ -946,9 +948,10 @@ def run_e2e(args, w, lres, hill, desc, mode, Kall, Vall, q_all, lens_all, k_all,
     return {"value": round(world * tokens / (ms / 1e3), 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": round(ms / len(order), 4),
             "api": calls + "; captured per decode step in a CUDA graph and replayed; every step copies one "
-                           "step's inputs in from pinned host memory and one step's results out to pinned host "
-                           "memory on a copy stream, overlapped with the compute (next step's inputs, previous "
-                           "step's results; two alternating buffer sets)",
+                           "step's inputs in from pinned host memory (writing its new K/V rows into the caches) "
+                           "and one step's results out to pinned host memory on a copy stream, overlapped with "
+                           "the compute (next step's inputs, previous step's results; two alternating buffer "
+                           "sets)",
             "eager": {"value": round(world * tokens / (ms_eager / 1e3), 1),
                       "ms_per_step": round(ms_eager / len(order), 4),
                       "api": calls + "; issued from Python at every step (no graph)"}}
