@@ -132,6 +132,40 @@ hill_status make_kmap8(const hill_desc* d, const void* k8, ScoreArgs* a) {
   return r == CUDA_SUCCESS ? HILL_OK : HILL_ERR_UNSUPPORTED;
 }
 
+// The same shadow for the tensor-core scoring: four maps whose boxes hold
+// 32, 64, 96 and 128 token rows (a chunk of one to four 32-token tiles).
+hill_status make_kmap8_tc(const hill_desc* d, const void* k8, ScoreTcArgs* a) {
+  auto fn = encode_tiled();
+  if (!fn) return HILL_ERR_CUDA;
+  const cuuint64_t cap = (cuuint64_t)std::max(d->capacity, 1), hkv = (cuuint64_t)d->num_kv_heads;
+  cuuint64_t gdim[4] = {(cuuint64_t)kHeadDim, cap, hkv, (cuuint64_t)std::max(d->batch, 1)};
+  cuuint64_t gstr[3] = {(cuuint64_t)kHeadDim, cap * kHeadDim, hkv * cap * kHeadDim};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  for (int m = 0; m < 4; ++m) {
+    cuuint32_t box[4] = {(cuuint32_t)kHeadDim, (cuuint32_t)(32 * (m + 1)), 1, 1};
+    CUresult r = fn(&a->kmap[m], CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<void*>(k8), gdim, gstr, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return HILL_ERR_UNSUPPORTED;
+  }
+  return HILL_OK;
+}
+
+// Tiled map of the query codes [rows][128] written by hill_quantize_q_kernel:
+// box = 128 codes x 16 rows (one KV head's query rows), 128-byte swizzle.
+hill_status make_qmap(const void* q8, int64_t rows, ScoreTcArgs* a) {
+  auto fn = encode_tiled();
+  if (!fn) return HILL_ERR_CUDA;
+  cuuint64_t gdim[2] = {(cuuint64_t)kHeadDim, (cuuint64_t)std::max<int64_t>(rows, 1)};
+  cuuint64_t gstr[1] = {(cuuint64_t)kHeadDim};
+  cuuint32_t box[2] = {(cuuint32_t)kHeadDim, (cuuint32_t)score_tc_max_group()};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(&a->qmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(q8), gdim, gstr, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? HILL_OK : HILL_ERR_UNSUPPORTED;
+}
+
 int cap32_of(const hill_desc* d) { return (d->capacity + 31) & ~31; }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -158,7 +192,7 @@ hill_status check_desc(const hill_desc* d) {
 }
 
 struct Layout {
-  size_t scores, logits, partials, stats, hist0, attn_part, total;
+  size_t scores, logits, partials, stats, hist0, attn_part, q8, sq, total;
   bool has_hist0;
   int score_grid, attn_grid, splits;
   int score_spc;   // ATTN partial slots per scoring CTA
@@ -182,9 +216,11 @@ int score_grid_for(const hill_desc* d, int sms, bool split_grid = false) {
 
 // Workspace regions of a call.  score_only: hill_score and its variants,
 // which write the caller's scores and run no selection or attention, need
-// only the ATTN normalisation's logits, partials and statistics.
+// only the ATTN normalisation's logits, partials and statistics.  e4m3_query:
+// room for the query codes and scales of the tensor-core E4M3 scoring (every
+// layout but the allocation-free entry point's, which scores 16-bit keys).
 Layout layout_for(const hill_desc* d, int mode, int max_k, int sms, bool score_only = false,
-                  bool split_grid = false) {
+                  bool split_grid = false, bool e4m3_query = true) {
   Layout L{};
   const size_t B = d->batch, H = d->num_q_heads, cap = d->capacity;
   L.score_grid = score_grid_for(d, sms, split_grid);
@@ -215,6 +251,11 @@ Layout layout_for(const hill_desc* d, int mode, int max_k, int sms, bool score_o
   if (L.has_hist0) off += align_up(B * (size_t)select_hist_bins() * sizeof(uint32_t));
   L.attn_part = off;
   off += align_up(B * H * (size_t)L.splits * (2 + kHeadDim) * sizeof(float));
+  // E4M3 query codes [B][Hkv][16][128] and scales [B][H]
+  L.q8 = off;
+  if (e4m3_query) off += align_up(B * (size_t)d->num_kv_heads * score_tc_max_group() * kHeadDim);
+  L.sq = off;
+  if (e4m3_query) off += align_up(B * H * sizeof(float));
   L.total = off + kAlign;  // room to align the caller's base pointer
   return L;
 }
@@ -308,8 +349,59 @@ hill_status run_score(const hill_desc* d, const void* q, const void* k, const in
   // or above the pass's heads (8 for the dealing kernel)
   const bool deal = L.score_spc > 1;
   a.Gs = G;
-  hill_status s = part == kScoreNormalise ? HILL_OK : head_passes(d, true, [&](int goff, int nkv, int hoff, int Gn,
-                                                                                bool first) {
+  // E4M3 scoring on the tensor cores' native 8-bit path (score_tc.cu) for
+  // per-sequence importance with 2 to 16 query heads per KV head (at most
+  // score_tc_max_heads() in all, one pass over the KV heads) and at least
+  // 64 MB of codes per call; measured against the warp-level kernel, in
+  // evaluation + selection per layer: one query head per KV head (4K and 32K
+  // MHA) 35.5 / 75.9 us there against 43.5 / 83.3 here; two heads (32K) 63.7
+  // against 50.4; four (32K, 128K) 39.9 / 45.5 against 36.8 / 35.9; four at
+  // 4K (34 MB of codes) 20.3 against 23.2.  Per-KV-head importance and the
+  // dealing layouts keep the warp-level kernel too.
+  const bool tc = f8 && !kvh && !deal && G >= 2 && G <= score_tc_max_group() &&
+                  d->num_kv_heads <= score_max_kv_heads() && d->num_q_heads <= score_tc_max_heads() &&
+                  (int64_t)d->batch * d->capacity * d->num_kv_heads * kHeadDim >= ((int64_t)64 << 20);
+  if (part != kScoreNormalise && tc) {
+    QuantQArgs qq{};
+    qq.q = q;
+    qq.q_sb = d->q_sb;
+    qq.q_sh = d->q_sh;
+    qq.B = d->batch;
+    qq.H = d->num_q_heads;
+    qq.Hkv = d->num_kv_heads;
+    qq.G = G;
+    qq.q8 = reinterpret_cast<uint8_t*>(base + L.q8);
+    qq.sq = reinterpret_cast<float*>(base + L.sq);
+    ScoreTcArgs t{};
+    hill_status ms = make_kmap8_tc(d, k, &t);
+    if (ms == HILL_OK) ms = make_qmap(qq.q8, (int64_t)d->batch * d->num_kv_heads * score_tc_max_group(), &t);
+    if (ms != HILL_OK) return ms;
+    t.kscale = kscale;
+    t.cap32 = cap32_of(d);
+    t.sq = qq.sq;
+    t.lens = lens;
+    t.B = d->batch;
+    t.H = d->num_q_heads;
+    t.Hkv = d->num_kv_heads;
+    t.cap = d->capacity;
+    t.G = G;
+    t.goff = 0;
+    t.nkv = d->num_kv_heads;
+    t.scores = a.scores;
+    t.accum = a.accum;
+    t.logits = a.logits;
+    t.lstride = a.lstride;
+    t.partials = a.partials;
+    t.nslot = a.nslot;
+    t.hist0 = a.hist0;
+    t.hist0_words = a.hist0_words;
+    t.err = a.err;
+    hill_status ts = from_cuda(counted(launch_quantize_q(qq, d->dtype, st), 1));
+    if (ts == HILL_OK) ts = from_cuda(counted(launch_score_tc(t, raw, L.score_grid, st), 1));
+    if (ts != HILL_OK || raw || part == kScoreStream) return ts;
+  }
+  hill_status s = part == kScoreNormalise || tc ? HILL_OK : head_passes(d, true, [&](int goff, int nkv, int hoff,
+                                                                                      int Gn, bool first) {
     a.goff = goff;
     a.nkv = nkv;
     a.hoff = hoff;
@@ -762,7 +854,7 @@ extern "C" hill_status hill_score_noalloc(const hill_desc* desc, const void* q, 
   if (!aligned16(q) || !aligned16(k_cache)) return HILL_ERR_INVALID_ARG;
   DeviceInfo di;
   if (device_info(&di) != cudaSuccess) return HILL_ERR_CUDA;
-  const Layout L = layout_for(desc, mode, 0, di.sms, true);
+  const Layout L = layout_for(desc, mode, 0, di.sms, true, false, false);
   // the array is already 256-byte aligned: the alignment slack is not needed
   if (L.total - kAlign > (size_t)HILL_SCORE_NOALLOC_MAX_SCRATCH) return HILL_ERR_WORKSPACE;
   void* scratch = nullptr;

@@ -59,6 +59,39 @@ struct FinalizeArgs {
   int tpt;            // blocks of 256 tokens per finalize CTA (set by the launcher)
 };
 
+// The E4M3 scoring on the tensor cores' native 8-bit path (score_tc.cu):
+// the K stream of ScoreArgs for E4M3 shadows, per-sequence ATTN or RAW, one
+// pass over at most score_max_kv_heads() KV heads with at most 16 query heads
+// each.
+struct ScoreTcArgs {
+  CUtensorMap kmap[4];   // codes [B][Hkv][cap][128]: 4-D maps (128, cap, Hkv, B), boxes of 128 codes x 32, 64, 96, 128 rows, 128-byte swizzle
+  CUtensorMap qmap;   // query codes [B*Hkv*16][128]: 2-D map, box 128 x 16 rows, 128-byte swizzle
+  const float* kscale;   // [B][Hkv][cap32] row scales
+  int cap32;
+  const float* sq;    // [B][H] query scales
+  const int32_t* lens;
+  int B, H, Hkv, cap, G, goff, nkv;
+  float* scores;      // RAW: per-token sums (may be NULL when accum is given)
+  float* accum;       // RAW: running importance (+=), may be NULL
+  float* logits;      // ATTN: [B][H][lstride]
+  int64_t lstride;
+  float2* partials;   // ATTN: [B][nslot][H] (max, sum 2^(z2 - max)), one slot per CTA meeting the sequence
+  int nslot;
+  uint32_t* hist0;    // optional: zero-filled here for the normalisation to count into
+  int64_t hist0_words;
+  unsigned* err;
+};
+
+// Query rows cast to E4M3 for the tensor-core scoring: q8[(b*Hkv + g)*16 + r]
+// holds query head g*G + r (rows r >= G zero), sq[b*H + h] its scale.
+struct QuantQArgs {
+  const void* q;
+  int64_t q_sb, q_sh;
+  int B, H, Hkv, G;
+  uint8_t* q8;
+  float* sq;
+};
+
 struct QuantArgs {
   const void* k;              // 16-bit K cache, strides k_sb, k_sh, k_sn
   const int32_t* row_begin;   // [B] rows [row_begin[b], row_end[b]) are quantised
@@ -165,6 +198,13 @@ cudaError_t launch_score(const ScoreArgs& a, int dtype, int G, bool raw, bool f8
 // which fits beside a scoring CTA on one SM.
 cudaError_t launch_attn_finalize(const FinalizeArgs& a, int sms, cudaStream_t st, int* kernels,
                                  bool two_kernel = false);
+
+// score_tc.cu
+int score_tc_tile_tokens();
+int score_tc_max_group();
+int score_tc_max_heads();
+cudaError_t launch_quantize_q(const QuantQArgs& a, int dtype, cudaStream_t st);
+cudaError_t launch_score_tc(const ScoreTcArgs& a, bool raw, int grid, cudaStream_t st);
 
 // selftest.cu
 cudaError_t launch_selftest_wait(unsigned long long limit_ns, unsigned* err, cudaStream_t st);

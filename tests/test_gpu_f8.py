@@ -2,7 +2,10 @@
 shadow written by hill_quantize_k (bit-exact against the oracle's float32
 quantisation), the scores of hill_score_f8 against the oracle's logits on the
 8-bit operands, and hill_evict_step_f8 (selection from the shadow, attention
-on the original 16-bit keys and values).
+on the original 16-bit keys and values).  The small shapes take the
+warp-level E4M3 kernel; TC_SHAPES (2 to 16 query heads per KV head, at least
+64 MB of codes) take the tensor-core kernel, through hill_score_f8 and the
+split step.
 """
 import numpy as np
 import pytest
@@ -108,6 +111,53 @@ def test_score_f8_matches_oracle(H, oracle_mod, mode, dtype, shape):
     codes, scale = oracle_mod.quantize_rows(K.cpu())
     z8 = oracle_mod.logits_q8(q.cpu(), codes, scale, lens)
     check_scores(s.cpu().numpy(), oracle_mod.scores(mode, z8, lens), lens)
+
+
+# Shapes that take the tensor-core E4M3 kernel (2 to 16 query heads per KV
+# head and at least 64 MB of codes per call): G = 4 on one 64K-token sequence,
+# G = 2 with two ragged sequences, G = 2 with three (one of a single token)
+TC_SHAPES = [
+    # B, H, Hkv, cap, lens
+    (1, 32, 8, 65600, [65537]),
+    (2, 32, 16, 33000, [33000, 20001]),
+    (3, 16, 8, 22000, [22000, 1, 15031]),
+]
+
+
+@pytest.mark.parametrize("mode", [ATTN, RAW])
+@pytest.mark.parametrize("dtype", [torch.float16, torch.bfloat16])
+@pytest.mark.parametrize("shape", TC_SHAPES, ids=lambda s: f"B{s[0]}H{s[1]}kv{s[2]}cap{s[3]}")
+def test_score_f8_tensor_core_matches_oracle(H, oracle_mod, mode, dtype, shape):
+    """hill_score_f8 and the split step's E4M3 K stream on shapes the
+    tensor-core kernel takes, against the oracle's scores on the 8-bit
+    operands; the split step's selection exact on its own scores."""
+    B, Hq, Hkv, cap, lens = shape
+    assert B * cap * Hkv * 128 >= 64 << 20
+    q, K, V, lens_t = inputs.random_case(B, Hq, Hkv, 128, cap, lens, dtype=dtype, seed=cap + 5 * Hq,
+                                         kind="zipf" if mode == ATTN else "normal")
+    q, K, lens_t = q.cuda(), K.cuda(), lens_t.cuda()
+    desc = H.make_desc(q, K)
+    k8, ks = _shadow(H, desc, K, lens)
+    codes, scale = oracle_mod.quantize_rows(K.cpu())
+    ref = oracle_mod.scores(mode, oracle_mod.logits_q8(q.cpu(), codes, scale, lens), lens)
+    ws = H.alloc_workspace(desc, mode, 0)
+    s = torch.full((B, cap), float("nan"), device="cuda")
+    H.hill_score_f8(desc, q, k8, ks, lens_t, mode, s, ws=ws)
+    H.hill_sync_status()
+    check_scores(s.cpu().numpy(), ref, lens)
+    k = [max(1, n // 10) for n in lens]
+    max_k = max(k)
+    wss = H.alloc_workspace(desc, mode, max_k)
+    s2 = torch.full((B, cap), float("nan"), device="cuda")
+    idx = torch.empty(B, max_k, dtype=torch.int32, device="cuda")
+    cnt = torch.empty(B, dtype=torch.int32, device="cuda")
+    kt = torch.tensor(k, dtype=torch.int32, device="cuda")
+    H.hill_evict_step_begin_f8(desc, q, k8, ks, lens_t, max_k, mode, None, s2, wss)
+    H.hill_evict_step_end(desc, lens_t, kt, max_k, mode, None, s2, idx, cnt, wss)
+    H.hill_sync_status()
+    check_scores(s2.cpu().numpy(), ref, lens, what="split step")
+    idx_o, cnt_o, _ = oracle_mod.topk(s2.cpu().numpy().astype(np.float64), lens, k, max_k)
+    assert np.array_equal(idx.cpu().numpy(), idx_o) and np.array_equal(cnt.cpu().numpy(), cnt_o)
 
 
 @pytest.mark.parametrize("mode", [ATTN, RAW])
