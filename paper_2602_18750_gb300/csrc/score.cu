@@ -62,7 +62,8 @@ struct ScoreCfg {
   static constexpr int kOffTab = kOffBar + kStages * 8;
   static constexpr int kOffRed = kOffTab + 2 * kTableInts * 4;
   static constexpr int kOffFlag = kOffRed + 2 * kNW * kT * 4;
-  static constexpr int kBytes = kOffFlag + kNW * 4 + 1024;   // + alignment slack
+  static constexpr int kOffIssued = kOffFlag + kNW * 4;       // warps that issued their last stage
+  static constexpr int kBytes = kOffIssued + 16 + 1024;   // + alignment slack
 };
 
 constexpr int kL2Ahead = 4;   // stages per warp brought into L2 before the dependency wait
@@ -121,6 +122,7 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
     for (int s = 0; s < kStages; ++s) mbar_init(base_addr + Cfg::kOffBar + s * 8, 1);
     fence_barrier_init();
     for (int w = 0; w < kNW; ++w) abort_flag[w] = 0;
+    *reinterpret_cast<int*>(base + Cfg::kOffIssued) = 0;
     prefetch_tmap(&a.kmap);
   }
   // Before the dependency wait this kernel reads only the inputs of the call
@@ -215,6 +217,16 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
   // prologue: the first kSW stages of this warp
   Cursor pc{it0, 0, b_first};
   uint32_t issued = 0, is_slot = 0;
+  // once every warp of the CTA has issued its last stage, the next kernel may
+  // launch (its CTAs take the SMs this grid's CTAs leave as they drain)
+  bool marked = false;
+  auto mark_if_done = [&]() {
+    if (!marked && (ng == 0 || pc.item >= it_hi)) {
+      marked = true;
+      if (lane == 0 && atomicAdd(reinterpret_cast<int*>(base + Cfg::kOffIssued), 1) == kNW - 1)
+        pdl_launch_dependents();
+    }
+  };
   auto prologue = [&]() {
     if (ng > 0) {
       for (; issued < (uint32_t)kSW && pc.item < it_hi; ++issued) {
@@ -243,10 +255,12 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
     }
   }
   pdl_wait();
-  // No early trigger: a dependent launches as these CTAs exit.  An early one
-  // would let the next layer's scoring grid (the next launch in this stream)
-  // take the SMs this grid leaves free for the normalisation and selection
-  // running beside it on another stream.
+  // No trigger here: a dependent launches once every CTA has issued its last
+  // stage (mark_if_done) or exited.  A trigger at the start would let the next
+  // layer's scoring grid (the next launch in this stream) take the SMs this
+  // grid leaves free for the normalisation and selection running beside it
+  // on another stream; one at the last issued stage lets it start on the SMs
+  // this grid's CTAs release as they drain.
   if (a.hist0) {   // this CTA's share of the leading-digit histogram, zeroed for the normalisation
     const int64_t hper = (a.hist0_words + gridDim.x - 1) / gridDim.x;
     const int64_t w0 = min((int64_t)blockIdx.x * hper, a.hist0_words);
@@ -255,6 +269,7 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
   }
   if (it_lo >= it_hi) return;
   if constexpr (F8) prologue();
+  mark_if_done();
 
   // fragment coordinates (mma.sync m16n8k16): C row = token lane/4 (+8),
   // C columns = heads 2*(lane%4) and 2*(lane%4)+1 of the group
@@ -445,6 +460,7 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
         }
         ++issued;
         advance(pc);
+        mark_if_done();
       }
 
       // the tile is scored for each fragment slot q: this stage's KV head
