@@ -217,9 +217,11 @@ __global__ void __maxnreg__(kScoreMaxRegs) hill_score_kernel(const __grid_consta
   // prologue: the first kSW stages of this warp
   Cursor pc{it0, 0, b_first};
   uint32_t issued = 0, is_slot = 0;
-  // once every warp of the CTA has issued its last stage, the next kernel may
-  // launch (its CTAs take the SMs this grid's CTAs leave as they drain)
-  bool marked = false;
+  // with 16-bit keys, once every warp of the CTA has issued its last stage the
+  // next kernel may launch (its CTAs take the SMs this grid's CTAs leave as
+  // they drain); the E4M3 path, whose loads wait for the shadow's row of this
+  // step, measured slower so and keeps the release at exit
+  bool marked = F8;
   auto mark_if_done = [&]() {
     if (!marked && (ng == 0 || pc.item >= it_hi)) {
       marked = true;
