@@ -200,7 +200,6 @@ cudaError_t launch_attn_finalize(const FinalizeArgs& a, int sms, cudaStream_t st
                                  bool two_kernel = false);
 
 // score_tc.cu
-int score_tc_tile_tokens();
 int score_tc_max_group();
 int score_tc_max_heads();
 cudaError_t launch_quantize_q(const QuantQArgs& a, int dtype, cudaStream_t st);

@@ -496,7 +496,6 @@ size_t tc_smem_bytes(int H) { return (size_t)kOffStats + (size_t)kTcPipes * H * 
 
 }  // namespace
 
-int score_tc_tile_tokens() { return kTcT; }
 int score_tc_max_group() { return kTcN; }
 int score_tc_max_heads() { return kTcMaxHeads; }
 
